@@ -1,0 +1,193 @@
+/*
+ * logo.h -- C ABI of the GB300 (sm_103a) LoGo attention hot path.
+ *
+ * LoGo (arXiv 2608.29539) gives every token sliding-window attention and lets
+ * a per-token gate send the selected tokens' queries, in addition, to full
+ * causal attention; the two normalised branch outputs are mixed by the gate.
+ * This library computes that layer's data-parallel path, forward and backward:
+ *
+ *   logo_select                  Eq. 7 threshold / per-sequence ratio, packing of I
+ *   logo_local_attn_fwd / _bwd   Eq. 6 local branch, window W, every token
+ *   logo_global_sparse_attn_fwd / _bwd
+ *                                Eq. 8 global branch on the selected rows only
+ *   logo_combine / _bwd          Eq. 9 ContextNorm + Eq. 10 gate-weighted fusion
+ *
+ * Conventions shared by every entry point
+ *   - All tensor pointers are DEVICE pointers owned by the caller.  The
+ *     library allocates no device memory: scratch comes from a caller
+ *     workspace of at least logo_*_workspace_size() bytes (16-byte aligned;
+ *     256-byte alignment recommended).
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream) and returns a status: LOGO_OK, or a negative LOGO_ERR_*
+ *     found on the host before anything was launched (bad argument, shape the
+ *     kernels do not support, launch failure).  Errors found on the device
+ *     (an expired bounded wait) are reported by logo_get_device_status().
+ *   - Layouts are row-major.  Q, K, V, O and their gradients are
+ *     [B, T, H, D] with H = Hq for queries/outputs and H = Hkv for keys and
+ *     values; bf16 tensors are passed as `logo_bf16` (raw bf16 bit patterns).
+ *     Query head h reads KV head h / (Hq / Hkv) (grouped-query attention).
+ *   - Positions are 0-based: token t of a sequence sees keys
+ *       local : s in [max(0, t - W + 1), t]   (Sec. 3.1, C^w_t, w keys with t)
+ *       global: s in [0, t]                   (Sec. 3.1, C^inf_t)
+ *   - Packed ("compacted") global rows follow App. B: the selected tokens of
+ *     sequence 0 in ascending position, then those of sequence 1, ...
+ *     Capacity is cap = B*T rows, so no call needs the count on the host.
+ *   - `scale` is the softmax temperature (Eq. 1 uses 1/sqrt(D)); pass 0 for
+ *     1/sqrt(D).  Softmax statistics `lse` are natural-log log-sum-exp values
+ *     of scale * q.k over the visible keys.
+ *   - Supported: D in {64, 128}; Hq % Hkv == 0; T >= 1; every tensor pointer
+ *     16-byte aligned and contiguous.
+ */
+#ifndef LOGO_H
+#define LOGO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define LOGO_API __attribute__((visibility("default")))
+#else
+#define LOGO_API
+#endif
+
+typedef uint16_t logo_bf16; /* bf16 bit pattern */
+
+#define LOGO_OK 0
+#define LOGO_ERR_INVALID_ARG (-1) /* null pointer, bad size, bad mode       */
+#define LOGO_ERR_UNSUPPORTED (-2) /* D not 64/128, Hq % Hkv != 0, misaligned */
+#define LOGO_ERR_CUDA (-3)        /* a CUDA runtime/driver call failed      */
+#define LOGO_ERR_TIMEOUT (-4)     /* device: a bounded wait expired         */
+#define LOGO_ERR_WORKSPACE (-5)   /* workspace missing or too small         */
+
+#define LOGO_SELECT_THRESHOLD 0 /* z_t = 1[p_t > b_th]                       */
+#define LOGO_SELECT_RATIO 1     /* top floor(ratio*T) gates per sequence     */
+
+typedef struct logo_dims {
+    int B;   /* sequences                        */
+    int T;   /* tokens per sequence              */
+    int Hq;  /* query heads                      */
+    int Hkv; /* key/value heads (Hq % Hkv == 0)  */
+    int D;   /* head dimension (64 or 128)       */
+} logo_dims;
+
+/* Reads and clears the device error word of every kernel of the library
+ * (synchronises the device).  *status receives LOGO_OK or the first
+ * LOGO_ERR_* a kernel recorded since the last call.  Returns LOGO_OK, or
+ * LOGO_ERR_CUDA if the word could not be read. */
+LOGO_API int logo_get_device_status(int* status);
+
+/* Number of SMs the persistent kernels size their grids for (device 0 of the
+ * current context); informational. */
+LOGO_API int logo_num_sms(void);
+
+/* ------------------------------------------------------------------------
+ * logo_select -- routing decision and packing of the selected set.
+ *   Eq. 7 (Sec. 3.2): z_t = 1[p_t > b_th], the gate p_t = sigmoid(x_t . w_g)
+ *   is computed by the caller; one decision per token, shared by all heads
+ *   (Sec. 3.1, after Eq. 2).  I = {t : z_t = 1} (Sec. 3.2), packed as in App. B.
+ *   mode LOGO_SELECT_THRESHOLD: strict float32 compare with b_th; b_th < 0
+ *     selects every token (the P-mask start of Sec. 3.2), b_th >= 1 none.
+ *   mode LOGO_SELECT_RATIO: in each sequence exactly k = floor(ratio * T)
+ *     tokens, those with the largest p_t; equal gates go to the lower position
+ *     (-0.0 and +0.0 compare equal).  ratio in [0, 1].  Gates must not be NaN.
+ * In : gate_p [B,T] float32.
+ * Out: z [B,T] uint8 (0/1); pos [B*T] int32 (in-sequence position of each
+ *      packed row; entries >= n_sel_total are left untouched); cu_q [B+1]
+ *      int32 (packed rows of sequence b are cu_q[b]..cu_q[b+1]); row_of [B,T]
+ *      int32 (packed row of a selected token, -1 otherwise); n_sel_total [1]
+ *      int32 (N = cu_q[B]; the realised ratio of Eq. 3 is N / (B*T)).
+ * Workspace: logo_select_workspace_size(dims) bytes.
+ * Integer outputs are bit-exact and deterministic. */
+LOGO_API size_t logo_select_workspace_size(logo_dims dims);
+LOGO_API int logo_select(const float* gate_p, logo_dims dims, int mode, float b_th, float ratio, uint8_t* z, int32_t* pos,
+                int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* workspace, size_t workspace_bytes,
+                void* stream);
+
+/* ------------------------------------------------------------------------
+ * logo_local_attn_fwd -- local branch O^L = SoftmaxAttn_W(Q^L, K^L, V^L)
+ *   (Eq. 6 with Eq. 1 over C^w_t), for all B*T tokens.  window >= 1;
+ *   window >= T is full causal attention.
+ * In : q [B,T,Hq,D], k/v [B,T,Hkv,D] bf16.
+ * Out: o [B,T,Hq,D] bf16; lse [B,Hq,T] float32 (kept for the backward).
+ * bf16 MMA on tcgen05 tensor cores with fp32 accumulation and softmax. */
+LOGO_API int logo_local_attn_fwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v, logo_bf16* o, float* lse,
+                        logo_dims dims, int window, float scale, void* stream);
+
+/* logo_local_attn_bwd -- gradients of logo_local_attn_fwd.
+ * In : q, k, v, o, lse as in/out of the forward; dO [B,T,Hq,D] bf16.
+ * Out: dq [B,T,Hq,D], dk/dv [B,T,Hkv,D] bf16 (overwritten; dk/dv sum over
+ *      the query heads of each group).
+ * Workspace: logo_local_attn_bwd_workspace_size(dims) bytes (fp32 dQ
+ * accumulator and row statistics). */
+LOGO_API size_t logo_local_attn_bwd_workspace_size(logo_dims dims);
+LOGO_API int logo_local_attn_bwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v, const logo_bf16* o,
+                        const float* lse, const logo_bf16* dO, logo_bf16* dq, logo_bf16* dk, logo_bf16* dv,
+                        logo_dims dims, int window, float scale, void* workspace, size_t workspace_bytes,
+                        void* stream);
+
+/* ------------------------------------------------------------------------
+ * logo_global_sparse_attn_fwd -- query-sparse global branch
+ *   O^G_I = SoftmaxAttn_inf(Q^G_I, K^G, V^G) (Eq. 8): only the packed
+ *   selected rows are computed, each against the dense causal prefix of its
+ *   real position (App. B), so every selected row gets exactly the dense
+ *   full-causal result.
+ * In : q [B,T,Hq,D] bf16 DENSE (rows gathered by pos inside the call);
+ *      k/v [B,T,Hkv,D] bf16; pos, cu_q, n_sel_total from logo_select.
+ * Out: o_c [B*T, Hq, D] bf16 packed (rows >= n_sel_total untouched);
+ *      lse_c [Hq, B*T] float32 packed.
+ * Workspace: logo_global_attn_fwd_workspace_size(dims) bytes (packed Q and
+ * the tile schedule). */
+LOGO_API size_t logo_global_attn_fwd_workspace_size(logo_dims dims);
+LOGO_API int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v, const int32_t* pos,
+                                const int32_t* cu_q, const int32_t* n_sel_total, logo_bf16* o_c, float* lse_c,
+                                logo_dims dims, float scale, void* workspace, size_t workspace_bytes,
+                                void* stream);
+
+/* logo_global_sparse_attn_bwd -- row-sparse backward of the global branch
+ *   (Sec. 3.3 and App. B): dQ only for selected rows, scattered to the dense
+ *   layout with zero rows for unselected tokens; dK/dV accumulate over the
+ *   selected rows that can see each key.
+ * In : q, k, v, pos, cu_q, n_sel_total as in the forward; o_c, lse_c from the
+ *      forward; dO_c [B*T, Hq, D] bf16 packed (rows < n_sel_total read).
+ * Out: dq [B,T,Hq,D] bf16 dense (zeros on unselected rows); dk/dv
+ *      [B,T,Hkv,D] bf16 (overwritten).
+ * Workspace: logo_global_attn_bwd_workspace_size(dims) bytes. */
+LOGO_API size_t logo_global_attn_bwd_workspace_size(logo_dims dims);
+LOGO_API int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v, const int32_t* pos,
+                                const int32_t* cu_q, const int32_t* n_sel_total, const logo_bf16* o_c,
+                                const float* lse_c, const logo_bf16* dO_c, logo_bf16* dq, logo_bf16* dk,
+                                logo_bf16* dv, logo_dims dims, float scale, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * logo_combine -- ContextNorm per branch (Eq. 9: head-wise RMSNorm over D,
+ *   r = 1/sqrt(mean_d o^2 + eps), o~ = o * r * gain) and the output fusion
+ *   (Eq. 10): o_t = (1 - p_t) o~L_t + p_t o~G_t if z_t = 1, else o~L_t.
+ * In : o_l [B,T,Hq,D] bf16; o_c [B*T,Hq,D] bf16 packed global rows; gate_p
+ *      [B,T] float32; z [B,T] uint8; row_of [B,T] int32; gain_l / gain_g
+ *      [Hq,D] float32 or NULL (= 1); eps > 0.
+ * Out: o [B,T,Hq,D] bf16; rstd_l [B,T,Hq] and rstd_g [B*T,Hq] float32 (the
+ *      RMS reciprocals r; either may be NULL). */
+LOGO_API int logo_combine(const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p, const uint8_t* z,
+                 const int32_t* row_of, const float* gain_l, const float* gain_g, float eps, logo_bf16* o,
+                 float* rstd_l, float* rstd_g, logo_dims dims, void* stream);
+
+/* logo_combine_bwd -- backward of logo_combine with z held fixed (z is a hard
+ *   indicator and passes no gradient):
+ *   do~L = dO (1 - p z), do~G = dO p, RMSNorm backward per branch, and
+ *   dp_t = z_t * sum_{h,d} dO (o~G - o~L).
+ * Out: dO_l [B,T,Hq,D] bf16; dO_c [B*T,Hq,D] bf16 packed (selected rows
+ *      written); dgate_p [B,T] float32 (0 on unselected tokens). */
+LOGO_API int logo_combine_bwd(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p,
+                     const uint8_t* z, const int32_t* row_of, const float* gain_l, const float* gain_g, float eps,
+                     logo_bf16* dO_l, logo_bf16* dO_c, float* dgate_p, logo_dims dims, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LOGO_H */

@@ -1,0 +1,572 @@
+// attn_fwd.cu -- forward of both attention branches on tcgen05 tensor cores.
+//
+//   logo_local_attn_fwd          O^L = SoftmaxAttn_W(Q^L, K^L, V^L)   (Eq. 6)
+//   logo_global_sparse_attn_fwd  O^G_I = SoftmaxAttn_inf(Q^G_I, K^G, V^G) (Eq. 8)
+//
+// One persistent kernel template serves both.  A CTA (6 warps) loops over
+// work items = (128-row query tile, query head):
+//   warp 0      TMA producer: Q tile once per item, then K/V blocks through a
+//               ring of shared-memory stages (128-byte swizzle).
+//   warp 1      MMA issuer (one thread): S = Q K^T into one of two TMEM S
+//               buffers, then O += P V into the TMEM O accumulator.
+//   warps 2..5  softmax: one thread per query row (its TMEM lane).  Online
+//               softmax in the log2 domain with conditional rescaling of O
+//               (only when the running max grows by more than 2^8); P is
+//               written to shared memory as bf16 for the P.V MMA.
+// The KV blocks of an item are only those some row can see; blocks where
+// every row sees every key skip the per-element predicate (App. B's
+// three-region traversal; for the local branch the window edge is a second
+// masked region).  Global items come from a schedule ordered by cost
+// (longest first) that a one-block kernel builds on the device, so nothing
+// here needs the selected count on the host.
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include "attn_common.cuh"
+#include "host_common.h"
+#include "sm100.cuh"
+
+namespace logo {
+namespace {
+
+template <int D>
+struct FwdCfg {
+    static constexpr int kSub = D / 64;                 // 64-column (128-byte) sub-tiles per row
+    static constexpr int kTileBytes = kBM * D * 2;      // one Q / K / V tile
+    static constexpr int kStages = (D == 128) ? 2 : 3;  // K/V ring depth
+    static constexpr int kPBytes = kBM * kBN * 2;
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffK = kOffQ + kTileBytes;
+    static constexpr int kOffV = kOffK + kStages * kTileBytes;
+    static constexpr int kOffP = kOffV + kStages * kTileBytes;
+    static constexpr int kSmemBytes = kOffP + kPBytes + 1024;  // + alignment slack
+    static constexpr uint32_t kColO = 0;
+    static constexpr uint32_t kColS0 = 128;
+    static constexpr uint32_t kColS1 = 256;
+    static constexpr uint32_t kTmemCols = 512;
+};
+
+struct FwdParams {
+    CUtensorMap tm_q;  // local: Q [B,T,Hq,D]; global: packed Qc [1,cap+128,Hq,D]
+    CUtensorMap tm_k;  // [B,T,Hkv,D]
+    CUtensorMap tm_v;
+    logo_bf16* o;      // local: [B,T,Hq,D]; global: packed [cap,Hq,D]
+    float* lse;        // local: [B,Hq,T];   global: [Hq,cap]
+    const int32_t* pos;            // global: packed positions
+    const GlobalTile* tiles;       // global: schedule
+    const int32_t* n_tiles;        // global: schedule length (device)
+    int B, T, Hq, Hkv, window, cap;
+    int q_tiles;                   // local: query tiles per sequence
+    float scale_log2;              // softmax scale * log2(e)
+};
+
+template <bool GLOBAL>
+__device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
+{
+    FwdItem it;
+    it.h = k % p.Hq;
+    it.kvh = it.h / (p.Hq / p.Hkv);
+    const int tile = k / p.Hq;
+    if (!GLOBAL) {
+        it.b = tile / p.q_tiles;
+        const int qt = tile % p.q_tiles;
+        it.row0 = qt * kBM;
+        it.nrows = min(kBM, p.T - it.row0);
+        it.pos_min = it.row0;
+        it.pos_max = it.row0 + it.nrows - 1;
+        it.blk_lo = max(0, it.pos_min - p.window + 1) / kBN;
+        it.blk_hi = it.pos_max / kBN;
+    } else {
+        const GlobalTile g = p.tiles[tile];
+        it.b = g.b;
+        it.row0 = g.row0;
+        it.nrows = g.nrows;
+        it.pos_min = g.min_pos;
+        it.pos_max = g.max_pos;
+        it.blk_lo = 0;
+        it.blk_hi = g.max_pos / kBN;
+    }
+    return it;
+}
+
+template <int D, bool GLOBAL>
+__global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
+{
+    using C = FwdCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_p_full, bar_o_done, bar_drain;
+    __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_v_full[C::kStages], bar_kv_empty[C::kStages];
+    __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2];
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ volatile int abort_flag;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t sQ = smem_u32(smem + C::kOffQ);
+    const uint32_t sK = smem_u32(smem + C::kOffK);
+    const uint32_t sV = smem_u32(smem + C::kOffV);
+    const uint32_t sP = smem_u32(smem + C::kOffP);
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        mbar_init(smem_u32(&bar_q_full), 1);
+        mbar_init(smem_u32(&bar_q_empty), 1);
+        mbar_init(smem_u32(&bar_p_full), 128);
+        mbar_init(smem_u32(&bar_o_done), 1);
+        mbar_init(smem_u32(&bar_drain), 1);
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(smem_u32(&bar_k_full[s]), 1);
+            mbar_init(smem_u32(&bar_v_full[s]), 1);
+            mbar_init(smem_u32(&bar_kv_empty[s]), 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(smem_u32(&bar_s_full[s]), 1);
+            mbar_init(smem_u32(&bar_s_empty[s]), 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(&tmem_base_sh), C::kTmemCols);
+        tmem_relinquish();
+    }
+    const int n_items = GLOBAL ? (*p.n_tiles) * p.Hq : p.B * p.q_tiles * p.Hq;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base_sh;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&p.tm_q);
+            tma_prefetch_desc(&p.tm_k);
+            tma_prefetch_desc(&p.tm_v);
+            const uint64_t pol_q = policy_evict_first();
+            const uint64_t pol_kv = policy_evict_last();
+            int kv_it = 0, item_i = 0;
+            int last_fill[C::kStages];
+            for (int s = 0; s < C::kStages; ++s) last_fill[s] = -1;
+            int q_fills = 0;
+            bool ok = true;
+            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x, ++item_i) {
+                const FwdItem it = decode_item<GLOBAL>(p, k);
+                if (!(ok = mbar_wait(smem_u32(&bar_q_empty), (item_i & 1) ^ 1, &abort_flag))) break;
+                const uint32_t qb = smem_u32(&bar_q_full);
+                mbar_arrive_expect_tx(qb, C::kTileBytes);
+                for (int s = 0; s < C::kSub; ++s)
+                    tma_load_4d(sQ + s * 16384, &p.tm_q, qb, 64 * s, it.h, it.row0, GLOBAL ? 0 : it.b, pol_q);
+                ++q_fills;
+                for (int n = it.blk_lo; n <= it.blk_hi; ++n, ++kv_it) {
+                    const int st = kv_it % C::kStages, f = kv_it / C::kStages;
+                    if (!(ok = mbar_wait(smem_u32(&bar_kv_empty[st]), (f & 1) ^ 1, &abort_flag))) break;
+                    const uint32_t kb = smem_u32(&bar_k_full[st]), vb = smem_u32(&bar_v_full[st]);
+                    mbar_arrive_expect_tx(kb, C::kTileBytes);
+                    for (int s = 0; s < C::kSub; ++s)
+                        tma_load_4d(sK + st * C::kTileBytes + s * 16384, &p.tm_k, kb, 64 * s, it.kvh, n * kBN, it.b,
+                                    pol_kv);
+                    mbar_arrive_expect_tx(vb, C::kTileBytes);
+                    for (int s = 0; s < C::kSub; ++s)
+                        tma_load_4d(sV + st * C::kTileBytes + s * 16384, &p.tm_v, vb, 64 * s, it.kvh, n * kBN, it.b,
+                                    pol_kv);
+                    last_fill[st] = f;
+                }
+            }
+            if (!ok) {  // let copies already issued land before the CTA exits
+                if (q_fills > 0) mbar_wait_drain(smem_u32(&bar_q_full), (q_fills - 1) & 1);
+                for (int s = 0; s < C::kStages; ++s)
+                    if (last_fill[s] >= 0) {
+                        mbar_wait_drain(smem_u32(&bar_k_full[s]), last_fill[s] & 1);
+                        mbar_wait_drain(smem_u32(&bar_v_full[s]), last_fill[s] & 1);
+                    }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, false, false);
+            constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, false, true);
+            int kv_it = 0, s_it = 0, item_i = 0;
+            bool ok = true;
+            auto issue_pv = [&](int jj) -> bool {
+                const int itg = s_it + jj;
+                const int st = (kv_it + jj) % C::kStages, f = (kv_it + jj) / C::kStages;
+                if (!mbar_wait(smem_u32(&bar_p_full), itg & 1, &abort_flag)) return false;
+                if (!mbar_wait(smem_u32(&bar_v_full[st]), f & 1, &abort_flag)) return false;
+                tc_fence_after();
+                const uint32_t vbase = sV + st * C::kTileBytes;
+#pragma unroll
+                for (int ks = 0; ks < kBN / 16; ++ks) {
+                    const uint64_t a = sdesc_sw128(sP + (ks >> 2) * 16384 + (ks & 3) * 32, 16, 1024);
+                    const uint64_t b = sdesc_sw128(vbase + ks * 2048, 16384, 1024);
+                    umma_bf16_ss(tmem + C::kColO, a, b, idPV, (jj > 0 || ks > 0) ? 1u : 0u);
+                }
+                umma_commit(smem_u32(&bar_o_done));
+                umma_commit(smem_u32(&bar_kv_empty[st]));
+                return true;
+            };
+            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x, ++item_i) {
+                const FwdItem it = decode_item<GLOBAL>(p, k);
+                const int nblk = it.blk_hi - it.blk_lo + 1;
+                if (!(ok = mbar_wait(smem_u32(&bar_q_full), item_i & 1, &abort_flag))) break;
+                for (int j = 0; j < nblk && ok; ++j) {
+                    const int itg = s_it + j;
+                    const int st = (kv_it + j) % C::kStages, f = (kv_it + j) / C::kStages;
+                    const int buf = itg & 1, use = itg >> 1;
+                    if (!(ok = mbar_wait(smem_u32(&bar_k_full[st]), f & 1, &abort_flag))) break;
+                    if (!(ok = mbar_wait(smem_u32(&bar_s_empty[buf]), (use & 1) ^ 1, &abort_flag))) break;
+                    tc_fence_after();
+                    const uint32_t kbase = sK + st * C::kTileBytes;
+                    const uint32_t dcol = tmem + (buf ? C::kColS1 : C::kColS0);
+#pragma unroll
+                    for (int ks = 0; ks < D / 16; ++ks) {
+                        const uint32_t off = (ks >> 2) * 16384 + (ks & 3) * 32;
+                        umma_bf16_ss(dcol, sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(kbase + off, 16, 1024), idS,
+                                     ks > 0 ? 1u : 0u);
+                    }
+                    umma_commit(smem_u32(&bar_s_full[buf]));
+                    if (j > 0) ok = issue_pv(j - 1);
+                }
+                if (!ok) break;
+                umma_commit(smem_u32(&bar_q_empty));
+                if (!(ok = issue_pv(nblk - 1))) break;
+                kv_it += nblk;
+                s_it += nblk;
+            }
+            if (!ok) {  // wait for MMAs in flight before TMEM is released
+                umma_commit(smem_u32(&bar_drain));
+                mbar_wait_drain(smem_u32(&bar_drain), 0);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ softmax
+        const int quad = warp & 3;  // TMEM lane quadrant this warp may access
+        const int r = quad * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        const int window = GLOBAL ? kNoWindow : p.window;
+        int itg = 0;
+        bool ok = true;
+        for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+            const FwdItem it = decode_item<GLOBAL>(p, k);
+            const bool row_valid = r < it.nrows;
+            int mypos;
+            if (GLOBAL) mypos = row_valid ? p.pos[it.row0 + r] : it.pos_max;
+            else mypos = row_valid ? it.row0 + r : it.pos_max;
+            float m_ref = -INFINITY;  // running max, log2 domain
+            float l = 0.f;
+            for (int n = it.blk_lo; n <= it.blk_hi; ++n, ++itg) {
+                const int buf = itg & 1, use = itg >> 1;
+                ok = mbar_wait(smem_u32(&bar_s_full[buf]), use & 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
+                float s[kBN];
+                const uint32_t scol = tmem + lane_off + (buf ? C::kColS1 : C::kColS0);
+#pragma unroll
+                for (int c = 0; c < kBN / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(scol + c * 32, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[i]);
+                }
+                tc_fence_before();
+                mbar_arrive(smem_u32(&bar_s_empty[buf]));
+                if (block_needs_mask(n, it.pos_min, it.pos_max, window)) {
+#pragma unroll
+                    for (int c = 0; c < kBN; ++c)
+                        if (!key_visible(n * kBN + c, mypos, window)) s[c] = -INFINITY;
+                }
+                float mx = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
+                const float m_new = fmaxf(m_ref, mx * p.scale_log2);
+                float alpha = 1.f;
+                bool rescale = false;
+                if (m_new > m_ref + 8.0f) {  // also taken when m_ref is still -inf
+                    alpha = ex2_approx(m_ref - m_new);
+                    m_ref = m_new;
+                    rescale = true;
+                }
+                const float m_use = (m_ref == -INFINITY) ? 0.f : m_ref;
+                float rs = 0.f;
+#pragma unroll
+                for (int c = 0; c < kBN; ++c) {
+                    s[c] = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
+                    rs += s[c];
+                }
+                l = l * alpha + rs;
+                // PV of the previous block must be done before O is rescaled
+                // or the P buffer is overwritten.
+                if (itg > 0) {
+                    ok = mbar_wait(smem_u32(&bar_o_done), (itg - 1) & 1, &abort_flag);
+                    __syncwarp();
+                    if (!ok) break;
+                    tc_fence_after();
+                }
+                // tcgen05.ld/st are warp-collective: rescale if any row of the
+                // warp needs it (the others multiply by alpha = 1).
+                if (__any_sync(0xffffffffu, rescale && n > it.blk_lo)) {
+                    const uint32_t ocol = tmem + lane_off + C::kColO;
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t v[32];
+                        tmem_ld32(ocol + c * 32, v);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                        tmem_st32(ocol + c * 32, v);
+                    }
+                    tmem_wait_st();
+                }
+#pragma unroll
+                for (int cc = 0; cc < kBN / 8; ++cc) {
+                    const uint32_t addr = sP + (cc >> 3) * 16384 + sw128_offset(r, cc & 7);
+                    st_shared_v4(addr, pack_bf16x2(s[8 * cc + 0], s[8 * cc + 1]), pack_bf16x2(s[8 * cc + 2], s[8 * cc + 3]),
+                                 pack_bf16x2(s[8 * cc + 4], s[8 * cc + 5]), pack_bf16x2(s[8 * cc + 6], s[8 * cc + 7]));
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(smem_u32(&bar_p_full));
+            }
+            if (!ok) break;
+            // ---- epilogue: O / l, lse = (m + log2 l) * ln 2
+            ok = mbar_wait(smem_u32(&bar_o_done), (itg - 1) & 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            tc_fence_after();
+            const float inv_l = 1.0f / l;
+            logo_bf16* orow;
+            if (GLOBAL) orow = p.o + (static_cast<int64_t>(it.row0 + r) * p.Hq + it.h) * D;
+            else orow = p.o + ((static_cast<int64_t>(it.b) * p.T + it.row0 + r) * p.Hq + it.h) * D;
+            const uint32_t ocol = tmem + lane_off + C::kColO;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(ocol + c * 32, v);
+                tmem_wait_ld();
+                if (row_valid) {
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(v[8 * q4 + 0]) * inv_l, __uint_as_float(v[8 * q4 + 1]) * inv_l);
+                        w.y = pack_bf16x2(__uint_as_float(v[8 * q4 + 2]) * inv_l, __uint_as_float(v[8 * q4 + 3]) * inv_l);
+                        w.z = pack_bf16x2(__uint_as_float(v[8 * q4 + 4]) * inv_l, __uint_as_float(v[8 * q4 + 5]) * inv_l);
+                        w.w = pack_bf16x2(__uint_as_float(v[8 * q4 + 6]) * inv_l, __uint_as_float(v[8 * q4 + 7]) * inv_l);
+                        *reinterpret_cast<uint4*>(orow + c * 32 + q4 * 8) = w;
+                    }
+                }
+            }
+            tc_fence_before();
+            if (row_valid) {
+                const float lse = (m_ref + log2f(l)) * kLn2;
+                if (GLOBAL) p.lse[static_cast<int64_t>(it.h) * p.cap + it.row0 + r] = lse;
+                else p.lse[(static_cast<int64_t>(it.b) * p.Hq + it.h) * p.T + it.row0 + r] = lse;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------- global prep
+// One block: split every sequence's packed rows into tiles of 128, and order
+// the tiles by their KV-block count, longest first.
+__global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __restrict__ pos,
+                                                               const int32_t* __restrict__ cu_q, int B,
+                                                               int32_t* __restrict__ tile_off,
+                                                               GlobalTile* __restrict__ unsorted,
+                                                               GlobalTile* __restrict__ sorted,
+                                                               int32_t* __restrict__ n_tiles)
+{
+    __shared__ int sh_nt;
+    if (threadIdx.x == 0) {
+        int acc = 0;
+        for (int b = 0; b < B; ++b) {
+            tile_off[b] = acc;
+            acc += (cu_q[b + 1] - cu_q[b] + kBM - 1) / kBM;
+        }
+        tile_off[B] = acc;
+        sh_nt = acc;
+        *n_tiles = acc;
+    }
+    __syncthreads();
+    const int nt = sh_nt;
+    for (int t = threadIdx.x; t < nt; t += blockDim.x) {
+        int lo = 0, hi = B - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (tile_off[mid] <= t) lo = mid;
+            else hi = mid - 1;
+        }
+        const int b = lo, i = t - tile_off[b];
+        GlobalTile g;
+        g.row0 = cu_q[b] + i * kBM;
+        g.nrows = min(kBM, cu_q[b + 1] - g.row0);
+        g.b = b;
+        g.min_pos = pos[g.row0];
+        g.max_pos = pos[g.row0 + g.nrows - 1];
+        g.pad0 = g.max_pos / kBN + 1;  // cost: KV blocks visited
+        g.pad1 = g.pad2 = 0;
+        unsorted[t] = g;
+    }
+    __syncthreads();
+    for (int t = threadIdx.x; t < nt; t += blockDim.x) {
+        const int c = unsorted[t].pad0;
+        int rank = 0;
+        for (int u = 0; u < nt; ++u) {
+            const int cu = unsorted[u].pad0;
+            rank += (cu > c) || (cu == c && u < t);
+        }
+        sorted[rank] = unsorted[t];
+    }
+}
+
+struct GlobalFwdWs {
+    logo_bf16* qc;
+    GlobalTile* unsorted;
+    GlobalTile* sorted;
+    int32_t* tile_off;
+    int32_t* n_tiles;
+};
+
+size_t global_fwd_ws_layout(const logo_dims& d, char* base, GlobalFwdWs* ws)
+{
+    const size_t cap = static_cast<size_t>(d.B) * d.T;
+    const size_t max_tiles = cap / kBM + d.B + 1;
+    size_t off = 0;
+    const size_t o_qc = off;
+    off = round_up(off + (cap + kBM) * d.Hq * d.D * 2, 256);
+    const size_t o_un = off;
+    off = round_up(off + max_tiles * sizeof(GlobalTile), 256);
+    const size_t o_so = off;
+    off = round_up(off + max_tiles * sizeof(GlobalTile), 256);
+    const size_t o_to = off;
+    off = round_up(off + (d.B + 1) * sizeof(int32_t), 256);
+    const size_t o_nt = off;
+    off = round_up(off + sizeof(int32_t), 256);
+    if (ws) {
+        ws->qc = reinterpret_cast<logo_bf16*>(base + o_qc);
+        ws->unsorted = reinterpret_cast<GlobalTile*>(base + o_un);
+        ws->sorted = reinterpret_cast<GlobalTile*>(base + o_so);
+        ws->tile_off = reinterpret_cast<int32_t*>(base + o_to);
+        ws->n_tiles = reinterpret_cast<int32_t*>(base + o_nt);
+    }
+    return off;
+}
+
+template <int D, bool GLOBAL>
+int launch_fwd(const FwdParams& prm, int n_items_upper, cudaStream_t st)
+{
+    using C = FwdCfg<D>;
+    static bool attr_done = false;  // benign race: setting the attribute twice is harmless
+    if (!attr_done) {
+        if (set_smem_limit(attn_fwd_kernel<D, GLOBAL>, C::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+        attr_done = true;
+    }
+    const int grid = max(1, min(n_items_upper, device_sm_count()));
+    attn_fwd_kernel<D, GLOBAL><<<grid, 192, C::kSmemBytes, st>>>(prm);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+int check_attn_ptrs(const void* q, const void* k, const void* v)
+{
+    if (!q || !k || !v) return LOGO_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v)) return LOGO_ERR_UNSUPPORTED;
+    return LOGO_OK;
+}
+
+}  // namespace
+
+int attn_fwd_tu_status(int clear) { return read_tu_status(clear); }
+
+}  // namespace logo
+
+using namespace logo;
+
+extern "C" int logo_local_attn_fwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v, logo_bf16* o,
+                                   float* lse, logo_dims dims, int window, float scale, void* stream)
+{
+    int rc = check_dims(dims);
+    if (rc != LOGO_OK) return rc;
+    if ((rc = check_attn_ptrs(q, k, v)) != LOGO_OK) return rc;
+    if (!o || !lse || window < 1) return LOGO_ERR_INVALID_ARG;
+    if (!aligned16(o)) return LOGO_ERR_UNSUPPORTED;
+    if (!(scale >= 0.0f)) return LOGO_ERR_INVALID_ARG;
+    if (scale == 0.0f) scale = 1.0f / sqrtf(static_cast<float>(dims.D));
+    FwdParams prm{};
+    const int w = window > dims.T ? dims.T : window;
+    if (!encode_bf16_4d(&prm.tm_q, q, dims.D, dims.Hq, dims.T, dims.B, 64, kBM) ||
+        !encode_bf16_4d(&prm.tm_k, k, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN) ||
+        !encode_bf16_4d(&prm.tm_v, v, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN))
+        return LOGO_ERR_CUDA;
+    prm.o = o;
+    prm.lse = lse;
+    prm.B = dims.B;
+    prm.T = dims.T;
+    prm.Hq = dims.Hq;
+    prm.Hkv = dims.Hkv;
+    prm.window = w;
+    prm.cap = dims.B * dims.T;
+    prm.q_tiles = (dims.T + kBM - 1) / kBM;
+    prm.scale_log2 = scale * kLog2e;
+    const int n_items = dims.B * prm.q_tiles * dims.Hq;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    return dims.D == 128 ? launch_fwd<128, false>(prm, n_items, st) : launch_fwd<64, false>(prm, n_items, st);
+}
+
+extern "C" size_t logo_global_attn_fwd_workspace_size(logo_dims dims)
+{
+    if (check_dims(dims) != LOGO_OK) return 0;
+    return global_fwd_ws_layout(dims, nullptr, nullptr);
+}
+
+extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* k, const logo_bf16* v,
+                                           const int32_t* pos, const int32_t* cu_q, const int32_t* n_sel_total,
+                                           logo_bf16* o_c, float* lse_c, logo_dims dims, float scale,
+                                           void* workspace, size_t workspace_bytes, void* stream)
+{
+    int rc = check_dims(dims);
+    if (rc != LOGO_OK) return rc;
+    if ((rc = check_attn_ptrs(q, k, v)) != LOGO_OK) return rc;
+    if (!pos || !cu_q || !n_sel_total || !o_c || !lse_c) return LOGO_ERR_INVALID_ARG;
+    if (!aligned16(o_c)) return LOGO_ERR_UNSUPPORTED;
+    if (!(scale >= 0.0f)) return LOGO_ERR_INVALID_ARG;
+    if (scale == 0.0f) scale = 1.0f / sqrtf(static_cast<float>(dims.D));
+    const size_t need = global_fwd_ws_layout(dims, nullptr, nullptr);
+    if (!workspace || workspace_bytes < need || !aligned16(workspace)) return LOGO_ERR_WORKSPACE;
+    GlobalFwdWs ws;
+    global_fwd_ws_layout(dims, static_cast<char*>(workspace), &ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int cap = dims.B * dims.T;
+    const int row_elems = dims.Hq * dims.D;
+    const int gather_grid = max(1, min(cap + kBM, device_sm_count() * 8));
+    gather_rows_kernel<<<gather_grid, 256, 0, st>>>(q, pos, cu_q, n_sel_total, dims.B, dims.T, row_elems, ws.qc);
+    global_schedule_kernel<<<1, 1024, 0, st>>>(pos, cu_q, dims.B, ws.tile_off, ws.unsorted, ws.sorted, ws.n_tiles);
+    if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    FwdParams prm{};
+    if (!encode_bf16_4d(&prm.tm_q, ws.qc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, kBM) ||
+        !encode_bf16_4d(&prm.tm_k, k, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN) ||
+        !encode_bf16_4d(&prm.tm_v, v, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN))
+        return LOGO_ERR_CUDA;
+    prm.o = o_c;
+    prm.lse = lse_c;
+    prm.pos = pos;
+    prm.tiles = ws.sorted;
+    prm.n_tiles = ws.n_tiles;
+    prm.B = dims.B;
+    prm.T = dims.T;
+    prm.Hq = dims.Hq;
+    prm.Hkv = dims.Hkv;
+    prm.window = kNoWindow;
+    prm.cap = cap;
+    prm.q_tiles = 0;
+    prm.scale_log2 = scale * kLog2e;
+    const int n_items_upper = static_cast<int>((static_cast<int64_t>(cap) / kBM + dims.B) * dims.Hq);
+    return dims.D == 128 ? launch_fwd<128, true>(prm, n_items_upper, st)
+                         : launch_fwd<64, true>(prm, n_items_upper, st);
+}

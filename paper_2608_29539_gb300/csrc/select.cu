@@ -1,0 +1,310 @@
+// select.cu -- logo_select: the routing decision of Eq. 7 (threshold mode) or
+// the per-sequence top-k reading of the target ratio (ratio mode), and the
+// stream compaction of the selected set I into the packed layout of App. B.
+//
+// Kernels (all on `stream`, no host synchronisation):
+//   radix_select_kernel  ratio mode only: per sequence, the k-th largest gate
+//                        key by 4 passes of 8-bit radix histograms; yields the
+//                        threshold key and how many tokens equal to it to take.
+//   count_kernel         per 1024-token chunk: tokens strictly selected and
+//                        (ratio mode) tokens tied with the threshold key.
+//   scan_kernel          one block: per-chunk output offsets, tie ranks,
+//                        cu_q[] and the total N.
+//   write_kernel         per chunk: block-wide prefix sums (warp ballots) turn
+//                        the decisions into z, pos and row_of, in ascending t.
+#include <cstdint>
+
+#include "host_common.h"
+#include "logo_status.cuh"
+
+namespace logo {
+namespace {
+
+constexpr int kChunk = 1024;     // tokens per chunk
+constexpr int kThreads = 256;    // threads per chunk block, 4 tokens each
+constexpr int kPerThread = kChunk / kThreads;
+
+// Order-preserving map of a float32 gate to uint32 (larger gate -> larger
+// key); -0.0 is folded onto +0.0 so the two compare equal, as floats do.
+__device__ __forceinline__ uint32_t gate_key(float p)
+{
+    uint32_t b = __float_as_uint(p);
+    if (b == 0x80000000u) b = 0u;
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+struct SeqThresh {
+    uint32_t key;   // tokens with key > this are selected
+    int need_eq;    // ... plus the first `need_eq` tokens with key == this
+};
+
+// Exclusive prefix sum over a 256-thread block; returns the exclusive value
+// and writes the block total to *total.
+__device__ __forceinline__ int block_excl_scan(int v, int* total, int* sh_warp)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh_warp[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        int w = (lane < kThreads / 32) ? sh_warp[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < kThreads / 32) sh_warp[lane] = w;  // inclusive warp totals
+    }
+    __syncthreads();
+    int base = (warp > 0) ? sh_warp[warp - 1] : 0;
+    *total = sh_warp[kThreads / 32 - 1];
+    __syncthreads();
+    return base + x - v;
+}
+
+// Ratio mode: find, per sequence, the key of the k-th largest gate.
+__global__ void __launch_bounds__(1024) radix_select_kernel(const float* __restrict__ p, int T, int k,
+                                                            SeqThresh* __restrict__ out)
+{
+    __shared__ int hist[256];
+    __shared__ uint32_t sh_prefix;
+    __shared__ int sh_remaining;
+    const int b = blockIdx.x;
+    const float* pb = p + static_cast<int64_t>(b) * T;
+    if (k <= 0) {
+        if (threadIdx.x == 0) out[b] = SeqThresh{0xFFFFFFFFu, 0};
+        return;
+    }
+    if (k >= T) {
+        if (threadIdx.x == 0) out[b] = SeqThresh{0u, T};
+        return;
+    }
+    uint32_t prefix = 0, mask = 0;
+    int remaining = k;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+        __syncthreads();
+        for (int t = threadIdx.x; t < T; t += blockDim.x) {
+            uint32_t key = gate_key(pb[t]);
+            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xFFu], 1);
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int above = 0;
+            int d = 255;
+            for (; d > 0; --d) {
+                if (above + hist[d] >= remaining) break;
+                above += hist[d];
+            }
+            sh_prefix = prefix | (static_cast<uint32_t>(d) << shift);
+            sh_remaining = remaining - above;
+        }
+        __syncthreads();
+        prefix = sh_prefix;
+        remaining = sh_remaining;
+        mask |= 0xFFu << shift;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) out[b] = SeqThresh{prefix, remaining};
+}
+
+struct ChunkCounts {
+    int gt;   // tokens selected outright in the chunk
+    int eq;   // tokens tied with the threshold key (ratio mode)
+};
+
+__device__ __forceinline__ void decide(float pv, bool ratio_mode, float b_th, const SeqThresh& th, bool* gt,
+                                       bool* eq)
+{
+    if (ratio_mode) {
+        uint32_t key = gate_key(pv);
+        *gt = key > th.key;
+        *eq = key == th.key;
+    } else {
+        *gt = pv > b_th;  // Eq. 7, strict
+        *eq = false;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) count_kernel(const float* __restrict__ p, int T, int nchunk,
+                                                         int ratio_mode, float b_th,
+                                                         const SeqThresh* __restrict__ th,
+                                                         ChunkCounts* __restrict__ counts)
+{
+    __shared__ int sh_warp[kThreads / 32];
+    const int c = blockIdx.x, b = blockIdx.y;
+    const int t0 = c * kChunk + threadIdx.x * kPerThread;
+    const float* pb = p + static_cast<int64_t>(b) * T;
+    SeqThresh tb = ratio_mode ? th[b] : SeqThresh{0u, 0};
+    int ngt = 0, neq = 0;
+#pragma unroll
+    for (int i = 0; i < kPerThread; ++i) {
+        int t = t0 + i;
+        if (t < T) {
+            bool gt, eq;
+            decide(pb[t], ratio_mode, b_th, tb, &gt, &eq);
+            ngt += gt;
+            neq += eq;
+        }
+    }
+    int tot_gt, tot_eq;
+    block_excl_scan(ngt, &tot_gt, sh_warp);
+    block_excl_scan(neq, &tot_eq, sh_warp);
+    if (threadIdx.x == 0) counts[static_cast<int64_t>(b) * nchunk + c] = ChunkCounts{tot_gt, tot_eq};
+}
+
+struct ChunkPlan {
+    int out_base;  // packed row of the chunk's first selected token
+    int eq_before; // tied tokens in earlier chunks of the same sequence
+};
+
+// One block: turns chunk counts into packed offsets (batch-major, ascending
+// t) and tie ranks; writes cu_q[0..B] and the total.
+__global__ void __launch_bounds__(kThreads) scan_kernel(const ChunkCounts* __restrict__ counts, int B, int nchunk,
+                                                        int ratio_mode, const SeqThresh* __restrict__ th,
+                                                        ChunkPlan* __restrict__ plan, int32_t* __restrict__ cu_q,
+                                                        int32_t* __restrict__ n_total)
+{
+    __shared__ int sh_warp[kThreads / 32];
+    int carry = 0;
+    for (int b = 0; b < B; ++b) {
+        if (threadIdx.x == 0) cu_q[b] = carry;
+        const int need = ratio_mode ? th[b].need_eq : 0;
+        int eq_carry = 0;
+        for (int c0 = 0; c0 < nchunk; c0 += kThreads) {
+            const int c = c0 + threadIdx.x;
+            ChunkCounts cc = (c < nchunk) ? counts[static_cast<int64_t>(b) * nchunk + c] : ChunkCounts{0, 0};
+            int eq_tot;
+            int eq_before = eq_carry + block_excl_scan(cc.eq, &eq_tot, sh_warp);
+            int take_eq = ratio_mode ? max(0, min(cc.eq, need - eq_before)) : 0;
+            int sel = cc.gt + take_eq;
+            int sel_tot;
+            int base = carry + block_excl_scan(sel, &sel_tot, sh_warp);
+            if (c < nchunk) plan[static_cast<int64_t>(b) * nchunk + c] = ChunkPlan{base, eq_before};
+            carry += sel_tot;
+            eq_carry += eq_tot;
+        }
+    }
+    if (threadIdx.x == 0) {
+        cu_q[B] = carry;
+        *n_total = carry;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) write_kernel(const float* __restrict__ p, int T, int nchunk,
+                                                         int ratio_mode, float b_th,
+                                                         const SeqThresh* __restrict__ th,
+                                                         const ChunkPlan* __restrict__ plan,
+                                                         uint8_t* __restrict__ z, int32_t* __restrict__ pos,
+                                                         int32_t* __restrict__ row_of)
+{
+    __shared__ int sh_warp[kThreads / 32];
+    const int c = blockIdx.x, b = blockIdx.y;
+    const int t0 = c * kChunk + threadIdx.x * kPerThread;
+    const int64_t off = static_cast<int64_t>(b) * T;
+    SeqThresh tb = ratio_mode ? th[b] : SeqThresh{0u, 0};
+    ChunkPlan pl = plan[static_cast<int64_t>(b) * nchunk + c];
+    bool gt[kPerThread], eq[kPerThread];
+    int neq = 0;
+#pragma unroll
+    for (int i = 0; i < kPerThread; ++i) {
+        int t = t0 + i;
+        gt[i] = eq[i] = false;
+        if (t < T) decide(p[off + t], ratio_mode, b_th, tb, &gt[i], &eq[i]);
+        neq += eq[i];
+    }
+    int tot;
+    int eq_rank = pl.eq_before + block_excl_scan(neq, &tot, sh_warp);
+    bool sel[kPerThread];
+    int nsel = 0;
+#pragma unroll
+    for (int i = 0; i < kPerThread; ++i) {
+        bool take = false;
+        if (eq[i]) {
+            take = eq_rank < tb.need_eq;
+            ++eq_rank;
+        }
+        sel[i] = gt[i] || take;
+        nsel += sel[i];
+    }
+    int row = pl.out_base + block_excl_scan(nsel, &tot, sh_warp);
+#pragma unroll
+    for (int i = 0; i < kPerThread; ++i) {
+        int t = t0 + i;
+        if (t < T) {
+            z[off + t] = sel[i] ? 1 : 0;
+            row_of[off + t] = sel[i] ? row : -1;
+            if (sel[i]) pos[row++] = t;
+        }
+    }
+}
+
+struct SelectWs {
+    SeqThresh* th;
+    ChunkCounts* counts;
+    ChunkPlan* plan;
+};
+
+size_t select_ws_layout(const logo_dims& d, char* base, SelectWs* ws)
+{
+    const size_t nchunk = (static_cast<size_t>(d.T) + kChunk - 1) / kChunk;
+    size_t off = 0;
+    size_t th_off = off;
+    off = round_up(off + sizeof(SeqThresh) * d.B, 256);
+    size_t cnt_off = off;
+    off = round_up(off + sizeof(ChunkCounts) * d.B * nchunk, 256);
+    size_t plan_off = off;
+    off = round_up(off + sizeof(ChunkPlan) * d.B * nchunk, 256);
+    if (ws) {
+        ws->th = reinterpret_cast<SeqThresh*>(base + th_off);
+        ws->counts = reinterpret_cast<ChunkCounts*>(base + cnt_off);
+        ws->plan = reinterpret_cast<ChunkPlan*>(base + plan_off);
+    }
+    return off;
+}
+
+}  // namespace
+
+int select_tu_status(int clear) { return read_tu_status(clear); }
+
+}  // namespace logo
+
+using namespace logo;
+
+extern "C" size_t logo_select_workspace_size(logo_dims dims)
+{
+    if (dims.B < 1 || dims.T < 1) return 0;
+    return select_ws_layout(dims, nullptr, nullptr);
+}
+
+extern "C" int logo_select(const float* gate_p, logo_dims dims, int mode, float b_th, float ratio, uint8_t* z,
+                           int32_t* pos, int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* workspace,
+                           size_t workspace_bytes, void* stream)
+{
+    if (dims.B < 1 || dims.T < 1) return LOGO_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(dims.B) * dims.T > (1ll << 30)) return LOGO_ERR_UNSUPPORTED;
+    if (!gate_p || !z || !pos || !cu_q || !row_of || !n_sel_total) return LOGO_ERR_INVALID_ARG;
+    if (mode != LOGO_SELECT_THRESHOLD && mode != LOGO_SELECT_RATIO) return LOGO_ERR_INVALID_ARG;
+    const bool ratio_mode = (mode == LOGO_SELECT_RATIO);
+    if (ratio_mode && !(ratio >= 0.0f && ratio <= 1.0f)) return LOGO_ERR_INVALID_ARG;
+    const size_t need = select_ws_layout(dims, nullptr, nullptr);
+    if (!workspace || workspace_bytes < need) return LOGO_ERR_WORKSPACE;
+    SelectWs ws;
+    select_ws_layout(dims, static_cast<char*>(workspace), &ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int nchunk = (dims.T + kChunk - 1) / kChunk;
+    // k = floor(rho * T), with rho read as float32 and the product in double
+    const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
+    if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
+    dim3 grid(nchunk, dims.B);
+    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.counts);
+    scan_kernel<<<1, kThreads, 0, st>>>(ws.counts, dims.B, nchunk, ratio_mode, ws.th, ws.plan, cu_q, n_sel_total);
+    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.plan, z, pos,
+                                            row_of);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}

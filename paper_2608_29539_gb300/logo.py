@@ -1,0 +1,258 @@
+"""Thin Python binding of the LoGo C ABI (``include/logo.h``).
+
+Argument marshalling only: every function here checks dtypes/shapes, allocates
+missing outputs and workspaces through torch (device memory is torch's job),
+and calls the entry point of the same name in ``_lib/liblogo.so`` on the
+current CUDA stream.  All computation runs in the library's CUDA kernels;
+there is no CPU path.  If the library has not been built, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+_c_int = ctypes.c_int
+_c_float = ctypes.c_float
+_c_size = ctypes.c_size_t
+_vp = ctypes.c_void_p
+
+LOGO_OK = 0
+LOGO_ERR_INVALID_ARG = -1
+LOGO_ERR_UNSUPPORTED = -2
+LOGO_ERR_CUDA = -3
+LOGO_ERR_TIMEOUT = -4
+LOGO_ERR_WORKSPACE = -5
+LOGO_SELECT_THRESHOLD = 0
+LOGO_SELECT_RATIO = 1
+
+_ERR_NAMES = {
+    LOGO_ERR_INVALID_ARG: "LOGO_ERR_INVALID_ARG",
+    LOGO_ERR_UNSUPPORTED: "LOGO_ERR_UNSUPPORTED",
+    LOGO_ERR_CUDA: "LOGO_ERR_CUDA",
+    LOGO_ERR_TIMEOUT: "LOGO_ERR_TIMEOUT",
+    LOGO_ERR_WORKSPACE: "LOGO_ERR_WORKSPACE",
+}
+
+
+class LogoError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} returned {_ERR_NAMES.get(code, code)}")
+        self.code = code
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [("B", _c_int), ("T", _c_int), ("Hq", _c_int), ("Hkv", _c_int), ("D", _c_int)]
+
+
+_lib = None
+
+_SIGS = {
+    "logo_get_device_status": (_c_int, [ctypes.POINTER(_c_int)]),
+    "logo_num_sms": (_c_int, []),
+    "logo_select_workspace_size": (_c_size, [Dims]),
+    "logo_select": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
+    "logo_local_attn_fwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp]),
+    "logo_local_attn_bwd_workspace_size": (_c_size, [Dims]),
+    "logo_local_attn_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp,
+                                     _c_size, _vp]),
+    "logo_global_attn_fwd_workspace_size": (_c_size, [Dims]),
+    "logo_global_sparse_attn_fwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_float, _vp, _c_size,
+                                             _vp]),
+    "logo_global_attn_bwd_workspace_size": (_c_size, [Dims]),
+    "logo_global_sparse_attn_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims,
+                                             _c_float, _vp, _c_size, _vp]),
+    "logo_combine": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_float, _vp, _vp, _vp, Dims, _vp]),
+    "logo_combine_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_float, _vp, _vp, _vp, Dims, _vp]),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load liblogo.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        path = _build.LIB
+        if not os.path.exists(path):
+            raise RuntimeError(f"LoGo CUDA library not built ({path}); run python -m paper_2608_29539_gb300.build")
+        L = ctypes.CDLL(path)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _p(t):
+    return None if t is None else _vp(t.data_ptr())
+
+
+def _stream():
+    return _vp(torch.cuda.current_stream().cuda_stream)
+
+
+def _call(name, *args):
+    rc = getattr(lib(), name)(*args)
+    if rc != LOGO_OK:
+        raise LogoError(name, rc)
+
+
+def _need(t, dtype, name, shape=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t
+
+
+def dims_of(q: torch.Tensor, k: torch.Tensor) -> Dims:
+    B, T, Hq, D = q.shape
+    return Dims(B, T, Hq, k.shape[2], D)
+
+
+def _workspace(nbytes: int, device, ws=None):
+    if ws is not None:
+        if ws.numel() * ws.element_size() < nbytes:
+            raise ValueError("workspace too small")
+        return ws
+    return torch.empty(max(int(nbytes), 16), dtype=torch.uint8, device=device)
+
+
+def workspace_bytes(kind: str, dims: Dims) -> int:
+    fn = {"select": "logo_select_workspace_size", "local_bwd": "logo_local_attn_bwd_workspace_size",
+          "global_fwd": "logo_global_attn_fwd_workspace_size",
+          "global_bwd": "logo_global_attn_bwd_workspace_size"}[kind]
+    return int(getattr(lib(), fn)(dims))
+
+
+# ----------------------------------------------------------------------- API
+def logo_get_device_status() -> int:
+    st = _c_int(0)
+    _call("logo_get_device_status", ctypes.byref(st))
+    return st.value
+
+
+def logo_num_sms() -> int:
+    return int(lib().logo_num_sms())
+
+
+def logo_select(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None, pos=None, cu_q=None,
+                row_of=None, n_sel_total=None, workspace=None):
+    """Eq. 7 routing and packing of I.  Returns (z, pos, cu_q, row_of, n_sel_total)."""
+    _need(gate_p, torch.float32, "gate_p")
+    B, T = gate_p.shape
+    dev = gate_p.device
+    dims = Dims(B, T, 1, 1, 64)
+    z = z if z is not None else torch.empty((B, T), dtype=torch.uint8, device=dev)
+    pos = pos if pos is not None else torch.empty((B * T,), dtype=torch.int32, device=dev)
+    cu_q = cu_q if cu_q is not None else torch.empty((B + 1,), dtype=torch.int32, device=dev)
+    row_of = row_of if row_of is not None else torch.empty((B, T), dtype=torch.int32, device=dev)
+    n_sel_total = n_sel_total if n_sel_total is not None else torch.empty((1,), dtype=torch.int32, device=dev)
+    nbytes = workspace_bytes("select", dims)
+    ws = _workspace(nbytes, dev, workspace)
+    _call("logo_select", _p(gate_p), dims, int(mode), float(b_th), float(ratio), _p(z), _p(pos), _p(cu_q),
+          _p(row_of), _p(n_sel_total), _p(ws), nbytes, _stream())
+    return z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_local_attn_fwd(q, k, v, window: int, scale: float = 0.0, o=None, lse=None):
+    """Eq. 6 local branch.  Returns (o [B,T,Hq,D] bf16, lse [B,Hq,T] fp32)."""
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _need(t, torch.bfloat16, n)
+    d = dims_of(q, k)
+    o = o if o is not None else torch.empty_like(q)
+    lse = lse if lse is not None else torch.empty((d.B, d.Hq, d.T), dtype=torch.float32, device=q.device)
+    _call("logo_local_attn_fwd", _p(q), _p(k), _p(v), _p(o), _p(lse), d, int(window), float(scale), _stream())
+    return o, lse
+
+
+def logo_local_attn_bwd(q, k, v, o, lse, dO, window: int, scale: float = 0.0, dq=None, dk=None, dv=None,
+                        workspace=None):
+    """Gradients of the local branch.  Returns (dq, dk, dv)."""
+    d = dims_of(q, k)
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (o, "o"), (dO, "dO")):
+        _need(t, torch.bfloat16, n)
+    _need(lse, torch.float32, "lse", (d.B, d.Hq, d.T))
+    dq = dq if dq is not None else torch.empty_like(q)
+    dk = dk if dk is not None else torch.empty_like(k)
+    dv = dv if dv is not None else torch.empty_like(v)
+    nbytes = workspace_bytes("local_bwd", d)
+    ws = _workspace(nbytes, q.device, workspace)
+    _call("logo_local_attn_bwd", _p(q), _p(k), _p(v), _p(o), _p(lse), _p(dO), _p(dq), _p(dk), _p(dv), d,
+          int(window), float(scale), _p(ws), nbytes, _stream())
+    return dq, dk, dv
+
+
+def logo_global_sparse_attn_fwd(q, k, v, pos, cu_q, n_sel_total, scale: float = 0.0, o_c=None, lse_c=None,
+                                workspace=None):
+    """Eq. 8 query-sparse global branch.  Returns (o_c [B*T,Hq,D], lse_c [Hq,B*T])."""
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _need(t, torch.bfloat16, n)
+    for t, n in ((pos, "pos"), (cu_q, "cu_q"), (n_sel_total, "n_sel_total")):
+        _need(t, torch.int32, n)
+    d = dims_of(q, k)
+    cap = d.B * d.T
+    o_c = o_c if o_c is not None else torch.empty((cap, d.Hq, d.D), dtype=torch.bfloat16, device=q.device)
+    lse_c = lse_c if lse_c is not None else torch.empty((d.Hq, cap), dtype=torch.float32, device=q.device)
+    nbytes = workspace_bytes("global_fwd", d)
+    ws = _workspace(nbytes, q.device, workspace)
+    _call("logo_global_sparse_attn_fwd", _p(q), _p(k), _p(v), _p(pos), _p(cu_q), _p(n_sel_total), _p(o_c),
+          _p(lse_c), d, float(scale), _p(ws), nbytes, _stream())
+    return o_c, lse_c
+
+
+def logo_global_sparse_attn_bwd(q, k, v, pos, cu_q, n_sel_total, o_c, lse_c, dO_c, scale: float = 0.0, dq=None,
+                                dk=None, dv=None, workspace=None):
+    """Row-sparse gradients of the global branch.  Returns (dq dense, dk, dv)."""
+    d = dims_of(q, k)
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (o_c, "o_c"), (dO_c, "dO_c")):
+        _need(t, torch.bfloat16, n)
+    _need(lse_c, torch.float32, "lse_c")
+    dq = dq if dq is not None else torch.empty_like(q)
+    dk = dk if dk is not None else torch.empty_like(k)
+    dv = dv if dv is not None else torch.empty_like(v)
+    nbytes = workspace_bytes("global_bwd", d)
+    ws = _workspace(nbytes, q.device, workspace)
+    _call("logo_global_sparse_attn_bwd", _p(q), _p(k), _p(v), _p(pos), _p(cu_q), _p(n_sel_total), _p(o_c),
+          _p(lse_c), _p(dO_c), _p(dq), _p(dk), _p(dv), d, float(scale), _p(ws), nbytes, _stream())
+    return dq, dk, dv
+
+
+def logo_combine(o_l, o_c, gate_p, z, row_of, gain_l=None, gain_g=None, eps: float = 1e-6, o=None, rstd_l=None,
+                 rstd_g=None):
+    """Eq. 9 ContextNorm + Eq. 10 fusion.  Returns (o, rstd_l, rstd_g)."""
+    _need(o_l, torch.bfloat16, "o_l")
+    _need(o_c, torch.bfloat16, "o_c")
+    B, T, H, D = o_l.shape
+    d = Dims(B, T, H, H, D)
+    o = o if o is not None else torch.empty_like(o_l)
+    rstd_l = rstd_l if rstd_l is not None else torch.empty((B, T, H), dtype=torch.float32, device=o_l.device)
+    rstd_g = rstd_g if rstd_g is not None else torch.empty((B * T, H), dtype=torch.float32, device=o_l.device)
+    _call("logo_combine", _p(o_l), _p(o_c), _p(gate_p), _p(z), _p(row_of), _p(gain_l), _p(gain_g), float(eps),
+          _p(o), _p(rstd_l), _p(rstd_g), d, _stream())
+    return o, rstd_l, rstd_g
+
+
+def logo_combine_bwd(dO, o_l, o_c, gate_p, z, row_of, gain_l=None, gain_g=None, eps: float = 1e-6, dO_l=None,
+                     dO_c=None, dgate_p=None):
+    """Backward of logo_combine with z fixed.  Returns (dO_l, dO_c, dgate_p)."""
+    _need(dO, torch.bfloat16, "dO")
+    B, T, H, D = o_l.shape
+    d = Dims(B, T, H, H, D)
+    dO_l = dO_l if dO_l is not None else torch.empty_like(o_l)
+    dO_c = dO_c if dO_c is not None else torch.empty((B * T, H, D), dtype=torch.bfloat16, device=o_l.device)
+    dgate_p = dgate_p if dgate_p is not None else torch.empty((B, T), dtype=torch.float32, device=o_l.device)
+    _call("logo_combine_bwd", _p(dO), _p(o_l), _p(o_c), _p(gate_p), _p(z), _p(row_of), _p(gain_l), _p(gain_g),
+          float(eps), _p(dO_l), _p(dO_c), _p(dgate_p), d, _stream())
+    return dO_l, dO_c, dgate_p

@@ -1,0 +1,85 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/logo.h declares; host-side argument checks reject bad calls before any
+CUDA work.  CPU only: nothing here launches a kernel."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_29539_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "logo.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^LOGO_API\s+\w+\s+(logo_\w+)\s*\(", text, flags=re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def test_header_declares_the_hot_path():
+    syms = declared_symbols()
+    for name in ("logo_select", "logo_local_attn_fwd", "logo_local_attn_bwd", "logo_global_sparse_attn_fwd",
+                 "logo_global_sparse_attn_bwd", "logo_combine", "logo_combine_bwd", "logo_get_device_status"):
+        assert name in syms
+
+
+def test_every_declared_symbol_is_exported(lib):
+    missing = [s for s in declared_symbols() if not hasattr(lib, s)]
+    assert not missing, missing
+
+
+def test_binding_covers_every_symbol():
+    from paper_2608_29539_gb300 import logo
+    assert set(declared_symbols()) == set(logo._SIGS)
+
+
+def test_host_side_argument_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    d = logo.Dims(1, 128, 2, 2, 128)
+    null = None
+    # null pointers
+    assert L.logo_select(null, d, 0, 0.5, 0.0, null, null, null, null, null, null, 0, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_local_attn_fwd(null, null, null, null, null, d, 64, 0.0, null) == logo.LOGO_ERR_INVALID_ARG
+    # unsupported head dim / grouping, invalid sizes
+    fake = ctypes.c_void_p(1 << 20)  # aligned, never dereferenced: rejected before use
+    for bad in (logo.Dims(1, 128, 2, 2, 96), logo.Dims(1, 128, 3, 2, 128)):
+        assert L.logo_local_attn_fwd(fake, fake, fake, fake, fake, bad, 64, 0.0, null) == logo.LOGO_ERR_UNSUPPORTED
+    assert L.logo_local_attn_fwd(fake, fake, fake, fake, fake, logo.Dims(0, 128, 2, 2, 128), 64, 0.0,
+                                 null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_local_attn_fwd(fake, fake, fake, fake, fake, d, 0, 0.0, null) == logo.LOGO_ERR_INVALID_ARG
+    # misaligned pointers
+    odd = ctypes.c_void_p((1 << 20) + 2)
+    assert L.logo_local_attn_fwd(odd, fake, fake, fake, fake, d, 64, 0.0, null) == logo.LOGO_ERR_UNSUPPORTED
+    # workspace too small
+    assert L.logo_global_sparse_attn_fwd(fake, fake, fake, fake, fake, fake, fake, fake, d, 0.0, fake, 16,
+                                         null) == logo.LOGO_ERR_WORKSPACE
+    assert L.logo_select(fake, d, 0, 0.5, 0.0, fake, fake, fake, fake, fake, fake, 0, null) == logo.LOGO_ERR_WORKSPACE
+    # bad mode / ratio
+    ws = L.logo_select_workspace_size(d)
+    assert L.logo_select(fake, d, 7, 0.5, 0.0, fake, fake, fake, fake, fake, fake, ws, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_select(fake, d, 1, 0.5, 1.5, fake, fake, fake, fake, fake, fake, ws, null) == logo.LOGO_ERR_INVALID_ARG
+    # combine: eps must be positive
+    assert L.logo_combine(fake, fake, fake, fake, fake, null, null, ctypes.c_float(0.0), fake, null, null, d,
+                          null) == logo.LOGO_ERR_INVALID_ARG
+
+
+def test_workspace_sizes_grow_with_shape(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    small, big = logo.Dims(1, 1024, 4, 4, 128), logo.Dims(2, 4096, 16, 16, 128)
+    for fn in ("logo_select_workspace_size", "logo_local_attn_bwd_workspace_size",
+               "logo_global_attn_fwd_workspace_size", "logo_global_attn_bwd_workspace_size"):
+        a, b = getattr(L, fn)(small), getattr(L, fn)(big)
+        assert 0 < a <= b, fn
+        if fn != "logo_select_workspace_size":
+            assert a < b, fn
+    assert L.logo_global_attn_fwd_workspace_size(logo.Dims(1, 128, 2, 2, 96)) == 0
