@@ -1,0 +1,468 @@
+#!/usr/bin/env python
+"""Benchmark of the LoGo attention layer's hot path on GB300.
+
+One step = one training pass of the layer over one batch of synthetic input:
+select -> local fwd -> global fwd -> combine -> combine bwd -> global bwd ->
+local bwd (every call through the C ABI, inputs resident in HBM).
+
+Metric: useful TFLOP/s of the whole step.  Useful FLOPs count only the
+query-key pairs the method must compute, 14*d per pair per head (4*d forward:
+Q.K^T and P.V; 10*d backward: S recompute, dP, dV, dQ, dK):
+  local pairs per head  = sum_t min(t+1, W)
+  global pairs per head = sum over selected t of (t+1)   (realised selection)
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Prints one JSON line (rank 0).  For N > 1 (torchrun) every rank runs its own
+replica of the workload (the path shards over sequences/heads with no
+exchange): value = all ranks' useful FLOPs / the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "LoGo attn fwd+bwd useful TFLOP/s & % bf16 TC peak, T=16K r=0.125"
+WORKLOAD = "16k"
+L2_BYTES = 129 * 1024 * 1024
+
+# DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by
+# the SHA-256 of the kernel source it was taken on; reported only while the
+# source is unchanged (see profiles/).
+TRAFFIC = {}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-dense", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ helpers
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm": float(p["hbm_gbs"]), "bf16": float(p["bf16_tflops"]),
+                "bf16_sus": float(p["bf16_tflops_sustained"]), "src": "measured"}
+    except Exception:
+        return {"hbm": 6800.0, "bf16": 1900.0, "bf16_sus": 1700.0, "src": "fallback"}
+
+
+def local_pairs(T, W):
+    W = min(W, T)
+    return W * (W + 1) // 2 + (T - W) * W
+
+
+def useful_flops(w, pos_by_seq):
+    lp = local_pairs(w.T, w.window) * w.B
+    gp = sum(int((p.astype(np.int64) + 1).sum()) for p in pos_by_seq)
+    per_pair = 14 * w.D * w.Hq
+    return lp * per_pair, gp * per_pair, lp, gp
+
+
+def src_hash(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={','.join(self.FIELDS)}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.idx)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ the step
+def make_device_inputs(w, device):
+    from paper_2608_29539_gb300.workloads import make_inputs
+    x = make_inputs(w, device=device)
+    return {k: v for k, v in x.items()}
+
+
+CALLS = ["select", "local_fwd", "global_fwd", "combine", "combine_bwd", "global_bwd", "local_bwd"]
+LAUNCHES_PER_STEP = {"select": 4, "local_fwd": 1, "global_fwd": 3, "combine": 1, "combine_bwd": 1,
+                     "global_bwd": 4, "local_bwd": 3}
+
+
+def run_step(layer, g, ev=None):
+    """One full step; if ev is given, record an event after each call."""
+    from paper_2608_29539_gb300 import logo as L
+    c = layer.cfg
+    if ev is not None:
+        ev[0].record()
+    L.logo_select(g["p"], c.mode, c.b_th, c.ratio, layer.z, layer.pos, layer.cu_q, layer.row_of, layer.n_sel,
+                  workspace=layer.ws)
+    if ev is not None:
+        ev[1].record()
+    L.logo_local_attn_fwd(g["qL"], g["kL"], g["vL"], c.window, c.scale, layer.o_l, layer.lse_l)
+    if ev is not None:
+        ev[2].record()
+    L.logo_global_sparse_attn_fwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q, layer.n_sel, c.scale,
+                                  layer.o_c, layer.lse_c, workspace=layer.ws)
+    if ev is not None:
+        ev[3].record()
+    L.logo_combine(layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of, None, None, c.eps, layer.o, layer.rstd_l,
+                   layer.rstd_g)
+    if ev is not None:
+        ev[4].record()
+    L.logo_combine_bwd(g["dO"], layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of, None, None, c.eps,
+                       layer.dO_l, layer.dO_c, layer.dgate)
+    if ev is not None:
+        ev[5].record()
+    L.logo_global_sparse_attn_bwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q, layer.n_sel, layer.o_c,
+                                  layer.lse_c, layer.dO_c, c.scale, layer.dqG, layer.dkG, layer.dvG,
+                                  workspace=layer.ws)
+    if ev is not None:
+        ev[6].record()
+    L.logo_local_attn_bwd(g["qL"], g["kL"], g["vL"], layer.o_l, layer.lse_l, layer.dO_l, c.window, c.scale,
+                          layer.dqL, layer.dkL, layer.dvL, workspace=layer.ws)
+    if ev is not None:
+        ev[7].record()
+
+
+def layer_for(w, device):
+    from paper_2608_29539_gb300 import logo as L
+    from paper_2608_29539_gb300.layer import LayerConfig, LogoAttention
+    mode = L.LOGO_SELECT_RATIO if w.mode == "ratio" else L.LOGO_SELECT_THRESHOLD
+    cfg = LayerConfig(w.B, w.T, w.Hq, w.Hkv, w.D, w.window, mode=mode, ratio=w.ratio)
+    return LogoAttention(cfg, device=device)
+
+
+def barrier(dist_on):
+    if dist_on:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, dist_on):
+    if not dist_on:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, dist_on):
+    if not dist_on:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ cpu side
+def oracle_sample(w, x, budget_s, pos_by_seq):
+    """Time the oracle on a bounded sample of the workload: the first
+    `nh` heads, the last `r` query rows of each branch of sequence 0 (the most
+    expensive rows), forward + backward.  Returns (useful TFLOP/s, seconds,
+    threads, description)."""
+    import oracle
+    nth = oracle.num_threads()
+    f = lambda t: t.detach().float().cpu().numpy()  # noqa: E731
+    qL, kL, vL = f(x["qL"][:1]), f(x["kL"][:1]), f(x["vL"][:1])
+    qG, kG, vG = f(x["qG"][:1]), f(x["kG"][:1]), f(x["vG"][:1])
+    group = w.Hq // w.Hkv
+    nh = max(group, min(w.Hq, (nth // group) * group))
+    heads = np.arange(nh, dtype=np.int32)
+    sel = pos_by_seq[0]
+    T = w.T
+
+    def run(r_local, r_global):
+        lt = np.arange(T - r_local, T, dtype=np.int32)
+        gt = sel[len(sel) - r_global:].astype(np.int32) if r_global else np.zeros(0, np.int32)
+        rng = np.random.default_rng(0)
+        t0 = time.perf_counter()
+        if r_local:
+            oracle.attn_fwd(qL, kL, vL, np.zeros_like(lt), lt, w.window, heads=heads)
+            dO = rng.standard_normal((r_local, w.Hq, w.D)).astype(np.float32)
+            oracle.attn_bwd(qL, kL, vL, np.zeros_like(lt), lt, w.window, dO, heads=heads)
+        if r_global:
+            oracle.attn_fwd(qG, kG, vG, np.zeros_like(gt), gt, 0, heads=heads)
+            dO = rng.standard_normal((r_global, w.Hq, w.D)).astype(np.float32)
+            oracle.attn_bwd(qG, kG, vG, np.zeros_like(gt), gt, 0, dO, heads=heads)
+        dt = time.perf_counter() - t0
+        pairs = sum(min(t + 1, w.window) for t in lt.tolist()) + int((gt.astype(np.int64) + 1).sum())
+        return dt, pairs * nh * 14 * w.D
+
+    r0 = 8
+    dt0, _ = run(r0, min(r0, len(sel)))
+    scale = max(1.0, budget_s / max(dt0, 1e-3))
+    r = int(min(T, r0 * scale))
+    rg = int(min(len(sel), r0 * scale))
+    dt, flops = run(r, rg)
+    desc = (f"oracle fp64 fwd+bwd on heads 0..{nh - 1} of sequence 0: the last {r} local query rows and the last "
+            f"{rg} selected global rows (the most expensive rows); useful FLOPs counted as on the GPU")
+    return flops / dt / 1e12, dt, nth, desc
+
+
+# ------------------------------------------------------------------ arms
+def reference_arm(a, rank, world):
+    """The oracle, as it stands, on the host cores: same metric and config."""
+    if rank != 0:
+        return
+    from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
+    import oracle
+    w = WORKLOADS[a.workload]
+    x = make_inputs(w, device="cpu")
+    p = x["p"].numpy()
+    z = oracle.select_ratio(p, w.k_per_seq) if w.mode == "ratio" else oracle.select_threshold(p, x["b_th"])
+    pos, cu_q, _, n = oracle.compact(z)
+    pos_by_seq = [pos[cu_q[b]:cu_q[b + 1]] for b in range(w.B)]
+    per_step = max(2.0, 150.0 / max(1, a.steps + a.warmup))
+    vals, secs = [], []
+    for i in range(a.warmup + a.steps):
+        v, dt, nth, desc = oracle_sample(w, x, per_step, pos_by_seq)
+        if i >= a.warmup:
+            vals.append(v)
+            secs.append(dt)
+    value = float(np.mean(vals))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": a.steps, "warmup": a.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_of(w),
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": nth, "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def config_of(w):
+    return {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} d={w.D} T={w.T} W={w.window} ratio={w.ratio} "
+                        f"({w.selection} selection), fwd+bwd",
+            "B": w.B, "T": w.T, "Hq": w.Hq, "Hkv": w.Hkv, "D": w.D, "window": w.window, "ratio": w.ratio,
+            "selection": w.selection, "mode": w.mode,
+            "l2": "inputs larger than L2 (6 x {:.0f} MiB bf16 Q/K/V tensors vs 129 MB L2); no flush".format(
+                w.B * w.T * w.Hq * w.D * 2 / 2**20)}
+
+
+def native_arm(a, rank, world, local_rank, dist_on):
+    from paper_2608_29539_gb300 import logo as L
+    from paper_2608_29539_gb300.workloads import WORKLOADS
+    w = WORKLOADS[a.workload]
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    pk = peaks()
+    x = make_device_inputs(w, "cuda")
+    layer = layer_for(w, dev)
+    run_step(layer, x)
+    torch.cuda.synchronize()
+    n = int(layer.n_sel.item())
+    cu = layer.cu_q.cpu().numpy()
+    pos = layer.pos[:n].cpu().numpy()
+    pos_by_seq = [pos[cu[b]:cu[b + 1]] for b in range(w.B)]
+    fl_local, fl_global, lp, gp = useful_flops(w, pos_by_seq)
+    fl_step = fl_local + fl_global
+
+    for _ in range(max(0, a.warmup - 1)):
+        run_step(layer, x)
+    # ---- timed region: K steps, per-call events on the launching stream
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(8)] for _ in range(a.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier(dist_on)
+    with ClockSampler(local_rank) as clk:
+        time.sleep(0.25)
+        t_start.record()
+        for s in range(a.steps):
+            run_step(layer, x, evs[s])
+        t_end.record()
+        torch.cuda.synchronize()
+        time.sleep(0.25)
+    barrier(dist_on)
+    st = L.logo_get_device_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the timed region")
+    total_ms = t_start.elapsed_time(t_end)
+    total_ms = max_over_ranks(total_ms, dist_on)
+    ms_step = total_ms / a.steps
+    per_call = {c: float(np.mean([evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(a.steps)]))
+                for i, c in enumerate(CALLS)}
+    flops_all = sum_over_ranks(fl_step * a.steps, dist_on)
+    value = flops_all / (total_ms / 1e3) / 1e12
+
+    # roofline of the dominant call (its tensor-core kernel dominates the call)
+    flops_call = {"local_fwd": fl_local * 4 / 14, "local_bwd": fl_local * 10 / 14,
+                  "global_fwd": fl_global * 4 / 14, "global_bwd": fl_global * 10 / 14}
+    dom = max(flops_call, key=lambda c: per_call[c])
+    achieved = flops_call[dom] / (per_call[dom] / 1e3) / 1e12
+    kernel_src = os.path.join(ROOT, "paper_2608_29539_gb300", "csrc",
+                              "attn_bwd.cu" if dom.endswith("bwd") else "attn_fwd.cu")
+    tr = TRAFFIC.get((dom, src_hash(kernel_src)))
+    roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+            "frac": achieved / pk["bf16_sus"], "traffic": tr,
+            "peak_note": f"{pk['src']} sustained bf16 (kernel timed inside a multi-ms step); "
+                         f"frac of burst peak {achieved / pk['bf16']:.3f}"}
+    g_ms = per_call["global_fwd"] + per_call["global_bwd"]
+    l_ms = per_call["local_fwd"] + per_call["local_bwd"]
+    breakdown = {c: {"ms": per_call[c]} for c in CALLS}
+    for c, fl in flops_call.items():
+        breakdown[c]["tflops"] = fl / (per_call[c] / 1e3) / 1e12
+    line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": a.steps,
+            "warmup": a.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; no dataset)", "config": config_of(w),
+            "frac_of_peak": value / pk["bf16_sus"],
+            "global_fwd_bwd": {"tflops": fl_global / (g_ms / 1e3) / 1e12,
+                               "frac_of_peak": fl_global / (g_ms / 1e3) / 1e12 / pk["bf16_sus"], "ms": g_ms},
+            "local_fwd_bwd": {"tflops": fl_local / (l_ms / 1e3) / 1e12, "ms": l_ms},
+            "useful_flops_per_step": fl_step, "pairs_per_head": {"local": lp, "global": gp},
+            "selected": n, "per_call": breakdown, "roofline": roof,
+            "gpu_launches": sum(LAUNCHES_PER_STEP.values()) * a.steps, "clocks": clk.summary()}
+
+    # ---- dense comparison: the same global kernels with every token selected
+    if not a.no_dense:
+        from paper_2608_29539_gb300.layer import LayerConfig, LogoAttention
+        dl = layer_for(w.with_(ratio=1.0), dev)
+        run_step(dl, x)
+        reps = 3
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(8)]
+        tt = []
+        for _ in range(reps):
+            run_step(dl, x, e)
+            torch.cuda.synchronize()
+            tt.append(e[2].elapsed_time(e[3]) + e[5].elapsed_time(e[6]))
+        dense_ms = float(np.median(tt))
+        dense_flops = w.B * w.T * (w.T + 1) // 2 * 14 * w.D * w.Hq
+        line["dense_global_fwd_bwd"] = {"ms": dense_ms, "tflops": dense_flops / (dense_ms / 1e3) / 1e12,
+                                        "speedup_sparse_vs_dense": dense_ms / g_ms,
+                                        "ideal_speedup": dense_flops / max(fl_global, 1)}
+        del dl
+
+    # ---- end to end through host buffers
+    if not a.no_e2e:
+        host = {k: x[k].cpu().pin_memory() for k in ("qL", "kL", "vL", "qG", "kG", "vG", "p", "dO")}
+        dev_in = {k: torch.empty_like(x[k]) for k in host}
+        out_o = torch.empty(layer.o.shape, dtype=layer.o.dtype).pin_memory()
+        out_dp = torch.empty(layer.dgate.shape, dtype=layer.dgate.dtype).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = out_o.numel() * out_o.element_size() + out_dp.numel() * out_dp.element_size()
+
+        def e2e_step():
+            for k in host:
+                dev_in[k].copy_(host[k], non_blocking=True)
+            run_step(layer, dev_in)
+            out_o.copy_(layer.o, non_blocking=True)
+            out_dp.copy_(layer.dgate, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(dist_on)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(a.steps):
+            e2e_step()
+        e1.record()
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist_on)
+        line["e2e"] = {"value": flops_all / (e2e_ms / 1e3) / 1e12, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                       "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / a.steps,
+                       "note": "pinned host inputs copied in and the layer output O plus dL/dp copied out each step"}
+    else:
+        line["e2e"] = None
+
+    # ---- the oracle on the host cores (rank 0, N = 1 only)
+    if rank == 0 and world == 1 and not a.no_cpu_baseline:
+        xc = {k: x[k][:1].cpu() for k in ("qL", "kL", "vL", "qG", "kG", "vG")}
+        v, dt, nth, desc = oracle_sample(w, xc, a.cpu_budget, pos_by_seq)
+        line["cpu_baseline"] = {"value": v, "unit": "TFLOP/s", "cores": nth, "kind": "oracle", "sample": desc,
+                                "seconds": dt}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    a = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    dist_on = world > 1
+    if dist_on:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        if a.impl == "reference":
+            reference_arm(a, rank, world)
+        else:
+            import __graft_entry__
+            __graft_entry__.build()
+            native_arm(a, rank, world, local_rank, dist_on)
+    finally:
+        if dist_on:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -312,3 +312,50 @@ def test_layer_step_4k_workload():
     check_close(np32(grads["dqG"])[:, :, h], dense[:, :, h], "dqG")
     check_close(np32(grads["dkG"])[:, :, h], rdk[:, :, h], "dkG")
     check_close(np32(grads["dvG"])[:, :, h], rdv[:, :, h], "dvG")
+
+
+# ------------------------------------------- full size, the benchmark's launch
+def test_full_size_16k_workload_sampled():
+    """The headline 16K workload (B=1, H=32, d=128, T=16384, W=1024, clustered
+    selection at ratio 1/8) through the same layer object bench.py times.
+    Selection checked in full; branch outputs on sampled rows of two heads;
+    combine in full; gradients in full for one head of each branch."""
+    import bench
+    from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
+    w = WORKLOADS["16k"]
+    x = make_inputs(w, device="cuda")
+    layer = bench.layer_for(w, torch.device("cuda"))
+    bench.run_step(layer, x)
+    torch.cuda.synchronize()
+    assert L().logo_get_device_status() == 0
+    n = int(layer.n_sel.item())
+    oz, opos, ocu, orow, on = oracle_select(x["p"].cpu(), 1, 0.0, w.ratio)
+    assert n == on == w.k_per_seq
+    np.testing.assert_array_equal(layer.pos[:n].cpu().numpy(), opos)
+    np.testing.assert_array_equal(layer.z.cpu().numpy(), oz)
+    np.testing.assert_array_equal(layer.row_of.cpu().numpy(), orow)
+    f = lambda k: np32(x[k])  # noqa: E731
+    qL, kL, vL, qG, kG, vG = (f(k) for k in ("qL", "kL", "vL", "qG", "kG", "vG"))
+    rng = np.random.default_rng(0)
+    heads = [0, 31]
+    rows = np.sort(np.concatenate([rng.choice(w.T, 200, replace=False), [0, 1, 1023, 1024, w.T - 1]]))
+    ro, _ = oracle.attn_fwd(qL, kL, vL, np.zeros_like(rows), rows, w.window, heads=heads)
+    check_close(np32(layer.o_l)[0, rows][:, heads], ro[:, heads], "o_l sampled")
+    grow = np.sort(np.concatenate([rng.choice(n, 200, replace=False), [0, n - 1]]))
+    rog, _ = oracle.attn_fwd(qG, kG, vG, np.zeros_like(grow), opos[grow], 0, heads=heads)
+    check_close(np32(layer.o_c)[grow][:, heads], rog[:, heads], "o_c sampled")
+    rfo, _, _ = oracle.combine_fwd(np32(layer.o_l), np32(layer.o_c)[:n], f("p"), oz, orow)
+    check_close(np32(layer.o), rfo, "o")
+    h = [7]
+    rb, rt = oracle.local_rows(w.B, w.T)
+    rdq, rdk, rdv = oracle.attn_bwd(qL, kL, vL, rb, rt, w.window, np32(layer.dO_l).reshape(-1, w.Hq, w.D), heads=h)
+    check_close(np32(layer.dqL).reshape(-1, w.Hq, w.D)[:, h], rdq[:, h], "dqL head 7")
+    check_close(np32(layer.dkL)[:, :, h], rdk[:, :, h], "dkL head 7")
+    check_close(np32(layer.dvL)[:, :, h], rdv[:, :, h], "dvL head 7")
+    gb, gt = oracle.global_rows(opos, ocu)
+    rdq, rdk, rdv = oracle.attn_bwd(qG, kG, vG, gb, gt, 0, np32(layer.dO_c)[:n], heads=h)
+    dense = np.zeros((w.B, w.T, w.Hq, w.D))
+    dense[gb, gt] = rdq
+    check_close(np32(layer.dqG)[:, :, h], dense[:, :, h], "dqG head 7")
+    check_close(np32(layer.dkG)[:, :, h], rdk[:, :, h], "dkG head 7")
+    check_close(np32(layer.dvG)[:, :, h], rdv[:, :, h], "dvG head 7")
