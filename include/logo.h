@@ -62,6 +62,7 @@ typedef uint16_t logo_bf16; /* bf16 bit pattern */
 #define LOGO_ERR_CUDA (-3)        /* a CUDA runtime/driver call failed      */
 #define LOGO_ERR_TIMEOUT (-4)     /* device: a bounded wait expired         */
 #define LOGO_ERR_WORKSPACE (-5)   /* workspace missing or too small         */
+#define LOGO_ERR_SCRATCH_LIMIT (-6) /* shape beyond a built-in scratch limit */
 
 #define LOGO_SELECT_THRESHOLD 0 /* z_t = 1[p_t > b_th]                       */
 #define LOGO_SELECT_RATIO 1     /* top floor(ratio*T) gates per sequence     */
@@ -106,6 +107,33 @@ LOGO_API size_t logo_select_workspace_size(logo_dims dims);
 LOGO_API int logo_select(const float* gate_p, logo_dims dims, int mode, float b_th, float ratio, uint8_t* z, int32_t* pos,
                 int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* workspace, size_t workspace_bytes,
                 void* stream);
+
+/* logo_select_noalloc -- logo_select for callers that cannot allocate.
+ *   No counterpart in the paper: this is a deployment variant of logo_select.
+ *   Some callers hold only their own input and output buffers and have no way
+ *   to obtain a workspace: a serving runtime that fixes all device memory
+ *   when it starts and forbids allocation per request, or a host in another
+ *   language that reaches this library through a plain C FFI without any
+ *   CUDA allocator of its own.  This entry point takes the same inputs and
+ *   outputs as logo_select (same results, bit for bit) and no workspace: its
+ *   scratch is a static device array of LOGO_SELECT_NOALLOC_SCRATCH_BYTES
+ *   inside the library, which every GPU that loads the library holds until the
+ *   process exits.  It calls no cudaMalloc, cudaFree or allocating routine.
+ *   Limits: B <= LOGO_SELECT_NOALLOC_MAX_SEQS and B * ceil(T / 1024) <=
+ *   LOGO_SELECT_NOALLOC_MAX_CHUNKS (at most 16,777,216 tokens per call);
+ *   larger shapes return LOGO_ERR_SCRATCH_LIMIT before anything is launched.
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current): make that first call
+ *   before any stream capture.  All calls share the one array, which keeps
+ *   the previous call's contents; every kernel writes the scratch it reads
+ *   before reading it, so no clearing is needed, but calls that overlap on
+ *   the GPU (different streams, or concurrent host threads) race on it and
+ *   must be serialised by the caller. */
+#define LOGO_SELECT_NOALLOC_MAX_SEQS 4096
+#define LOGO_SELECT_NOALLOC_MAX_CHUNKS 16384
+#define LOGO_SELECT_NOALLOC_SCRATCH_BYTES 294912
+LOGO_API int logo_select_noalloc(const float* gate_p, logo_dims dims, int mode, float b_th, float ratio, uint8_t* z,
+                                 int32_t* pos, int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* stream);
 
 /* ------------------------------------------------------------------------
  * logo_local_attn_fwd -- local branch O^L = SoftmaxAttn_W(Q^L, K^L, V^L)

@@ -13,6 +13,7 @@
 //   write_kernel         per chunk: block-wide prefix sums (warp ballots) turn
 //                        the decisions into z, pos and row_of, in ascending t.
 #include <cstdint>
+#include <mutex>
 
 #include "host_common.h"
 #include "logo_status.cuh"
@@ -299,6 +300,65 @@ extern "C" int logo_select(const float* gate_p, logo_dims dims, int mode, float 
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int nchunk = (dims.T + kChunk - 1) / kChunk;
     // k = floor(rho * T), with rho read as float32 and the product in double
+    const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
+    if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
+    dim3 grid(nchunk, dims.B);
+    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.counts);
+    scan_kernel<<<1, kThreads, 0, st>>>(ws.counts, dims.B, nchunk, ratio_mode, ws.th, ws.plan, cu_q, n_sel_total);
+    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.plan, z, pos,
+                                            row_of);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------------------
+// logo_select_noalloc: the same kernels with their scratch in a static device
+// array instead of a caller workspace (for callers that cannot allocate).
+namespace logo {
+namespace {
+
+static __device__ __align__(256) unsigned char g_select_noalloc_scratch[LOGO_SELECT_NOALLOC_SCRATCH_BYTES];
+
+// Device address of the array, looked up once per device (the name is only a
+// host-side stand-in and must never be passed to a kernel).
+int noalloc_scratch_ptr(char** out)
+{
+    static std::mutex mu;
+    static void* cached[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return LOGO_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cached[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_select_noalloc_scratch) != cudaSuccess || !p) return LOGO_ERR_CUDA;
+        cached[dev] = p;
+    }
+    *out = static_cast<char*>(cached[dev]);
+    return LOGO_OK;
+}
+
+}  // namespace
+}  // namespace logo
+
+extern "C" int logo_select_noalloc(const float* gate_p, logo_dims dims, int mode, float b_th, float ratio,
+                                   uint8_t* z, int32_t* pos, int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total,
+                                   void* stream)
+{
+    if (dims.B < 1 || dims.T < 1) return LOGO_ERR_INVALID_ARG;
+    if (!gate_p || !z || !pos || !cu_q || !row_of || !n_sel_total) return LOGO_ERR_INVALID_ARG;
+    if (mode != LOGO_SELECT_THRESHOLD && mode != LOGO_SELECT_RATIO) return LOGO_ERR_INVALID_ARG;
+    const bool ratio_mode = (mode == LOGO_SELECT_RATIO);
+    if (ratio_mode && !(ratio >= 0.0f && ratio <= 1.0f)) return LOGO_ERR_INVALID_ARG;
+    const int64_t nchunk64 = (static_cast<int64_t>(dims.T) + kChunk - 1) / kChunk;
+    if (dims.B > LOGO_SELECT_NOALLOC_MAX_SEQS || dims.B * nchunk64 > LOGO_SELECT_NOALLOC_MAX_CHUNKS)
+        return LOGO_ERR_SCRATCH_LIMIT;
+    if (select_ws_layout(dims, nullptr, nullptr) > sizeof(g_select_noalloc_scratch)) return LOGO_ERR_SCRATCH_LIMIT;
+    char* scratch = nullptr;
+    int rc = noalloc_scratch_ptr(&scratch);
+    if (rc != LOGO_OK) return rc;
+    SelectWs ws;
+    select_ws_layout(dims, scratch, &ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int nchunk = static_cast<int>(nchunk64);
     const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
     if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
     dim3 grid(nchunk, dims.B);

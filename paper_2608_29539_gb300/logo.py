@@ -26,6 +26,7 @@ LOGO_ERR_UNSUPPORTED = -2
 LOGO_ERR_CUDA = -3
 LOGO_ERR_TIMEOUT = -4
 LOGO_ERR_WORKSPACE = -5
+LOGO_ERR_SCRATCH_LIMIT = -6
 LOGO_SELECT_THRESHOLD = 0
 LOGO_SELECT_RATIO = 1
 
@@ -35,6 +36,7 @@ _ERR_NAMES = {
     LOGO_ERR_CUDA: "LOGO_ERR_CUDA",
     LOGO_ERR_TIMEOUT: "LOGO_ERR_TIMEOUT",
     LOGO_ERR_WORKSPACE: "LOGO_ERR_WORKSPACE",
+    LOGO_ERR_SCRATCH_LIMIT: "LOGO_ERR_SCRATCH_LIMIT",
 }
 
 
@@ -55,6 +57,7 @@ _SIGS = {
     "logo_num_sms": (_c_int, []),
     "logo_select_workspace_size": (_c_size, [Dims]),
     "logo_select": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
+    "logo_select_noalloc": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp]),
     "logo_local_attn_fwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp]),
     "logo_local_attn_bwd_workspace_size": (_c_size, [Dims]),
     "logo_local_attn_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp,
@@ -163,6 +166,26 @@ def logo_select(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None
     ws = _workspace(nbytes, dev, workspace)
     _call("logo_select", _p(gate_p), dims, int(mode), float(b_th), float(ratio), _p(z), _p(pos), _p(cu_q),
           _p(row_of), _p(n_sel_total), _p(ws), nbytes, _stream())
+    return z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_select_noalloc(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None, pos=None, cu_q=None,
+                        row_of=None, n_sel_total=None):
+    """logo_select without a workspace, for callers that cannot allocate
+    scratch (its scratch is a static device array inside the library; see
+    include/logo.h for the size limits).  The outputs must be given or are
+    allocated here by torch.  Returns (z, pos, cu_q, row_of, n_sel_total)."""
+    _need(gate_p, torch.float32, "gate_p")
+    B, T = gate_p.shape
+    dev = gate_p.device
+    dims = Dims(B, T, 1, 1, 64)
+    z = z if z is not None else torch.empty((B, T), dtype=torch.uint8, device=dev)
+    pos = pos if pos is not None else torch.empty((B * T,), dtype=torch.int32, device=dev)
+    cu_q = cu_q if cu_q is not None else torch.empty((B + 1,), dtype=torch.int32, device=dev)
+    row_of = row_of if row_of is not None else torch.empty((B, T), dtype=torch.int32, device=dev)
+    n_sel_total = n_sel_total if n_sel_total is not None else torch.empty((1,), dtype=torch.int32, device=dev)
+    _call("logo_select_noalloc", _p(gate_p), dims, int(mode), float(b_th), float(ratio), _p(z), _p(pos), _p(cu_q),
+          _p(row_of), _p(n_sel_total), _stream())
     return z, pos, cu_q, row_of, n_sel_total
 
 
