@@ -424,6 +424,441 @@ __global__ void __launch_bounds__(192, 1) attn_bwd_kernel(const __grid_constant_
     }
 }
 
+// ---------------------------------------------------------------- d = 128
+// Overlapped variant for D = 128: query tiles of 64 rows with two TMEM
+// buffers, so the MMAs of tile u+1 (S^T, dP^T) run while the softmax warps
+// work on tile u, and dQ is produced transposed (dQ^T = K^T dS^T, one TMEM lane
+// per head-dim row) into the columns S^T of that tile occupied.  Roles:
+//   warp 0       TMA: K/V per item, Q/dO tiles through a 3-deep ring
+//   warp 1       MMA issuer: S^T, dP^T (M=128 keys, N=64 queries) into buffer
+//                u%2; then, once P^T/dS^T of tile u-1 are in shared memory,
+//                dV += P^T dO, dK += dS^T Q, dQ^T = K^T dS^T
+//   warps 2..9   two warpgroups, one per 32-query half of the tile; thread =
+//                key row: P^T and dS^T (bf16) from S^T and dP^T
+//   warps 10..13 dQ^T out of TMEM (thread = head-dim row), coalesced fp32
+//                atomics into the dQ accumulator (one 128-byte row segment per
+//                warp instruction); dK/dV epilogue at the end of each item
+struct Bwd2Cfg {
+    static constexpr int D = 128;
+    static constexpr int kBQ = 64;                 // queries per tile
+    static constexpr int kStages = 3;              // Q/dO ring depth
+    static constexpr int kKVBytes = kBN * D * 2;   // K or V block: 32 KB
+    static constexpr int kQBytes = kBQ * D * 2;    // Q or dO tile: 16 KB (two 8 KB halves of d)
+    static constexpr int kPBytes = kBN * kBQ * 2;  // P^T or dS^T: 16 KB
+    static constexpr int kOffK = 0;
+    static constexpr int kOffV = kOffK + kKVBytes;
+    static constexpr int kOffQ = kOffV + kKVBytes;
+    static constexpr int kOffDO = kOffQ + kStages * kQBytes;
+    static constexpr int kOffP = kOffDO + kStages * kQBytes;  // 2 buffers
+    static constexpr int kOffDS = kOffP + 2 * kPBytes;        // 2 buffers
+    static constexpr int kSmemBytes = kOffDS + 2 * kPBytes + 1024;
+    static constexpr uint32_t kColDK = 0;
+    static constexpr uint32_t kColDV = 128;
+    static constexpr uint32_t kColBuf = 256;  // buffer b: S^T at 256+128b (64 cols), dP^T at +64
+    static constexpr uint32_t kTmemCols = 512;
+    static constexpr int kThreads = 448;
+};
+
+template <bool GLOBAL>
+__device__ __forceinline__ BwdItem decode_bwd2(const BwdParams& p, int k)
+{
+    BwdItem it;
+    it.kvh = k % p.Hkv;
+    const int t = k / p.Hkv;
+    it.b = t % p.B;
+    it.j = t / p.B;
+    const int k0 = it.j * kBN;
+    constexpr int BQ = Bwd2Cfg::kBQ;
+    if (!GLOBAL) {
+        it.i_lo = k0 / BQ;
+        const int i_hi = min((p.T + BQ - 1) / BQ - 1, (k0 + kBN - 1 + p.window - 1) / BQ);
+        it.ntiles = i_hi - it.i_lo + 1;
+        it.row_lo = it.row_hi = 0;
+    } else {
+        it.row_lo = p.cu_q[it.b];
+        it.row_hi = p.cu_q[it.b + 1];
+        int lo = it.row_lo, hi = it.row_hi;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (p.pos[mid] < k0) lo = mid + 1;
+            else hi = mid;
+        }
+        if (lo >= it.row_hi) {
+            it.i_lo = 0;
+            it.ntiles = 0;
+        } else {
+            it.i_lo = lo / BQ;
+            it.ntiles = (it.row_hi - 1) / BQ - it.i_lo + 1;
+        }
+    }
+    return it;
+}
+
+template <bool GLOBAL>
+__global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const __grid_constant__ BwdParams p)
+{
+    using C = Bwd2Cfg;
+    constexpr int D = C::D, BQ = C::kBQ, NS = C::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t bar_kv_full, bar_kv_empty, bar_dkv_full, bar_dkv_empty, bar_drain, bar_stage;
+    __shared__ __align__(8) uint64_t bar_qdo_full[NS], bar_qdo_empty[NS];
+    __shared__ __align__(8) uint64_t bar_st_full[2], bar_ds_full[2], bar_dq_full[2], bar_dq_empty[2];
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ volatile int abort_flag;
+    __shared__ int sh_pos[2][BQ];
+    __shared__ float2 sh_ld[2][BQ];     // (lse in log2 units, Dsum) per query column
+    __shared__ int sh_open[2][2];       // per staging warp: every column sees every key of the block
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t sK = smem_u32(smem + C::kOffK), sV = smem_u32(smem + C::kOffV);
+    const uint32_t sQ = smem_u32(smem + C::kOffQ), sDO = smem_u32(smem + C::kOffDO);
+    const uint32_t sP = smem_u32(smem + C::kOffP), sDS = smem_u32(smem + C::kOffDS);
+    const int group = p.Hq / p.Hkv;
+    const int n_items = p.B * p.nblk * p.Hkv;
+
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        mbar_init(smem_u32(&bar_kv_full), 1);
+        mbar_init(smem_u32(&bar_kv_empty), 1);
+        mbar_init(smem_u32(&bar_dkv_full), 1);
+        mbar_init(smem_u32(&bar_dkv_empty), 128);
+        mbar_init(smem_u32(&bar_drain), 1);
+        mbar_init(smem_u32(&bar_stage), 256);
+        for (int s = 0; s < NS; ++s) {
+            mbar_init(smem_u32(&bar_qdo_full[s]), 1);
+            mbar_init(smem_u32(&bar_qdo_empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&bar_st_full[b]), 1);
+            mbar_init(smem_u32(&bar_ds_full[b]), 256);
+            mbar_init(smem_u32(&bar_dq_full[b]), 1);
+            mbar_init(smem_u32(&bar_dq_empty[b]), 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(&tmem_base_sh), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base_sh;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&p.tm_q);
+            tma_prefetch_desc(&p.tm_do);
+            tma_prefetch_desc(&p.tm_k);
+            tma_prefetch_desc(&p.tm_v);
+            const uint64_t pol_q = policy_evict_last();
+            const uint64_t pol_kv = policy_evict_first();
+            int u = 0, kv_items = 0;
+            bool ok = true;
+            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+                const BwdItem it = decode_bwd2<GLOBAL>(p, k);
+                if (it.ntiles == 0) continue;
+                if (!(ok = mbar_wait(smem_u32(&bar_kv_empty), (kv_items & 1) ^ 1, &abort_flag))) break;
+                const uint32_t kvb = smem_u32(&bar_kv_full);
+                mbar_arrive_expect_tx(kvb, 2 * C::kKVBytes);
+                for (int s = 0; s < 2; ++s) {
+                    tma_load_4d(sK + s * 16384, &p.tm_k, kvb, 64 * s, it.kvh, it.j * kBN, it.b, pol_kv);
+                    tma_load_4d(sV + s * 16384, &p.tm_v, kvb, 64 * s, it.kvh, it.j * kBN, it.b, pol_kv);
+                }
+                ++kv_items;
+                const int n_it = group * it.ntiles;
+                for (int x = 0; x < n_it; ++x, ++u) {
+                    const int h = it.kvh * group + x / it.ntiles;
+                    const int i = it.i_lo + x % it.ntiles;
+                    const int st = u % NS, f = u / NS;
+                    if (!(ok = mbar_wait(smem_u32(&bar_qdo_empty[st]), (f & 1) ^ 1, &abort_flag))) break;
+                    const uint32_t qb = smem_u32(&bar_qdo_full[st]);
+                    mbar_arrive_expect_tx(qb, 2 * C::kQBytes);
+                    const int cb = GLOBAL ? 0 : it.b;
+                    for (int s = 0; s < 2; ++s) {
+                        tma_load_4d(sQ + st * C::kQBytes + s * 8192, &p.tm_q, qb, 64 * s, h, i * BQ, cb, pol_q);
+                        tma_load_4d(sDO + st * C::kQBytes + s * 8192, &p.tm_do, qb, 64 * s, h, i * BQ, cb, pol_q);
+                    }
+                }
+            }
+            if (!ok) {  // let copies already issued land before the CTA exits
+                if (kv_items > 0) mbar_wait_drain(smem_u32(&bar_kv_full), (kv_items - 1) & 1);
+                for (int v = u - NS > 0 ? u - NS : 0; v < u; ++v)
+                    mbar_wait_drain(smem_u32(&bar_qdo_full[v % NS]), (v / NS) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16_f32(kBN, BQ, false, false);  // S^T, dP^T: 128 x 64
+            constexpr uint32_t idKV = idesc_bf16_f32(kBN, D, false, true);   // dV, dK: 128 x 128
+            constexpr uint32_t idQ = idesc_bf16_f32(D, BQ, true, true);      // dQ^T: 128 x 64
+            int u = 0, kv_items = 0;
+            bool ok = true;
+            // second half of tile v: dV, dK, dQ^T (x_in_item: position of v in its item)
+            auto issue_b = [&](int v, int x_in_item) -> bool {
+                const int b = v & 1, st = v % NS;
+                if (!mbar_wait(smem_u32(&bar_ds_full[b]), (v >> 1) & 1, &abort_flag)) return false;
+                if (x_in_item == 0 && !mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))
+                    return false;
+                tc_fence_after();
+                const uint32_t pb = sP + b * C::kPBytes, db = sDS + b * C::kPBytes;
+                const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
+#pragma unroll
+                for (int ks = 0; ks < BQ / 16; ++ks) {
+                    const uint32_t acc = (x_in_item > 0 || ks > 0) ? 1u : 0u;
+                    umma_bf16_ss(tmem + C::kColDV, sdesc_sw128(pb + ks * 32, 16, 1024),
+                                 sdesc_sw128(ob + ks * 2048, 8192, 1024), idKV, acc);
+                    umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
+                                 sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
+                }
+#pragma unroll
+                for (int ks = 0; ks < kBN / 16; ++ks) {
+                    umma_bf16_ss(tmem + C::kColBuf + 128 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
+                                 sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
+                }
+                umma_commit(smem_u32(&bar_dq_full[b]));
+                umma_commit(smem_u32(&bar_qdo_empty[st]));
+                return true;
+            };
+            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+                const BwdItem it = decode_bwd2<GLOBAL>(p, k);
+                if (it.ntiles == 0) continue;
+                if (!(ok = mbar_wait(smem_u32(&bar_kv_full), kv_items & 1, &abort_flag))) break;
+                const int n_it = group * it.ntiles;
+                for (int x = 0; x < n_it; ++x, ++u) {
+                    const int b = u & 1, st = u % NS;
+                    if (!(ok = mbar_wait(smem_u32(&bar_qdo_full[st]), (u / NS) & 1, &abort_flag))) break;
+                    if (!(ok = mbar_wait(smem_u32(&bar_dq_empty[b]), ((u >> 1) & 1) ^ 1, &abort_flag))) break;
+                    tc_fence_after();
+                    const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
+                    const uint32_t scol = tmem + C::kColBuf + 128 * b;
+#pragma unroll
+                    for (int ks = 0; ks < D / 16; ++ks) {
+                        const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;
+                        const uint32_t kb = (ks >> 2) * 8192 + (ks & 3) * 32;
+                        umma_bf16_ss(scol, sdesc_sw128(sK + ka, 16, 1024), sdesc_sw128(qb + kb, 16, 1024), idS,
+                                     ks > 0 ? 1u : 0u);
+                    }
+#pragma unroll
+                    for (int ks = 0; ks < D / 16; ++ks) {
+                        const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;
+                        const uint32_t kb = (ks >> 2) * 8192 + (ks & 3) * 32;
+                        umma_bf16_ss(scol + 64, sdesc_sw128(sV + ka, 16, 1024), sdesc_sw128(ob + kb, 16, 1024), idS,
+                                     ks > 0 ? 1u : 0u);
+                    }
+                    umma_commit(smem_u32(&bar_st_full[b]));
+                    if (x > 0 && !(ok = issue_b(u - 1, x - 1))) break;
+                }
+                if (!ok) break;
+                if (!(ok = issue_b(u - 1, n_it - 1))) break;
+                umma_commit(smem_u32(&bar_kv_empty));
+                umma_commit(smem_u32(&bar_dkv_full));
+                ++kv_items;
+            }
+            if (!ok) {
+                umma_commit(smem_u32(&bar_drain));
+                mbar_wait_drain(smem_u32(&bar_drain), 0);
+            }
+        }
+    } else if (warp < 10) {
+        // ------------------------------------------------------------ P^T, dS^T
+        const int quad = warp & 3;
+        const int half = (warp - 2) >> 2;   // query columns half*32 .. half*32+31
+        const int t = quad * 32 + lane;     // key row of the block
+        const int tw = threadIdx.x - 64;    // 0..255 across both warpgroups
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        const int window = GLOBAL ? kNoWindow : p.window;
+        int u = 0;
+        bool ok = true;
+        for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+            const BwdItem it = decode_bwd2<GLOBAL>(p, k);
+            if (it.ntiles == 0) continue;
+            const int k0 = it.j * kBN;
+            const int key = k0 + t;
+            const int n_it = group * it.ntiles;
+            for (int x = 0; x < n_it; ++x, ++u) {
+                const int h = it.kvh * group + x / it.ntiles;
+                const int i = it.i_lo + x % it.ntiles;
+                const int b = u & 1;
+                if (tw < BQ) {  // stage the tile's query positions, lse (log2 units), Dsum
+                    int pc = -1;
+                    float2 ld = make_float2(0.f, 0.f);
+                    bool open = false;  // this column sees every key of the block
+                    if (!GLOBAL) {
+                        const int q = i * BQ + tw;
+                        if (q < p.T) {
+                            const int64_t idx = (static_cast<int64_t>(it.b) * p.Hq + h) * p.T + q;
+                            pc = q;
+                            ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
+                            open = q >= k0 + kBN - 1 && q - k0 < window;
+                        }
+                    } else {
+                        const int row = i * BQ + tw;
+                        if (row >= it.row_lo && row < it.row_hi) {
+                            const int64_t idx = static_cast<int64_t>(h) * p.cap + row;
+                            pc = p.pos[row];
+                            ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
+                            open = pc >= k0 + kBN - 1;
+                        }
+                    }
+                    sh_pos[b][tw] = pc;
+                    sh_ld[b][tw] = ld;
+                    const bool all_open = __all_sync(0xffffffffu, open);
+                    if (lane == 0) sh_open[b][tw >> 5] = all_open ? 1 : 0;
+                }
+                mbar_arrive(smem_u32(&bar_stage));
+                ok = mbar_wait(smem_u32(&bar_stage), u & 1, &abort_flag);
+                if (!ok) break;
+                const bool open = sh_open[b][0] && sh_open[b][1];
+                ok = mbar_wait(smem_u32(&bar_st_full[b]), (u >> 1) & 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                // P^T / dS^T buffer b is free once the MMAs of tile u-2 are done
+                // (they were issued before S^T of tile u, so this rarely waits)
+                ok = mbar_wait(smem_u32(&bar_dq_full[b]), ((u >> 1) & 1) ^ 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
+                uint32_t sv[32], dpv[32];
+                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + half * 32, sv);
+                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + 64 + half * 32, dpv);
+                tmem_wait_ld();
+                uint32_t pk[16], dk2[16];
+                if (open) {
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        float pe[2], de[2];
+#pragma unroll
+                        for (int zz = 0; zz < 2; ++zz) {
+                            const float2 ld = sh_ld[b][half * 32 + e + zz];
+                            const float pr = ex2_approx(fmaf(__uint_as_float(sv[e + zz]), p.scale_log2, -ld.x));
+                            pe[zz] = pr;
+                            de[zz] = pr * (__uint_as_float(dpv[e + zz]) - ld.y);
+                        }
+                        pk[e / 2] = pack_bf16x2(pe[0], pe[1]);
+                        dk2[e / 2] = pack_bf16x2(de[0], de[1]);
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        float pe[2], de[2];
+#pragma unroll
+                        for (int zz = 0; zz < 2; ++zz) {
+                            const int c = half * 32 + e + zz;
+                            const float2 ld = sh_ld[b][c];
+                            const bool vis = key_visible(key, sh_pos[b][c], window);
+                            const float pr =
+                                vis ? ex2_approx(fmaf(__uint_as_float(sv[e + zz]), p.scale_log2, -ld.x)) : 0.f;
+                            pe[zz] = pr;
+                            de[zz] = pr * (__uint_as_float(dpv[e + zz]) - ld.y);
+                        }
+                        pk[e / 2] = pack_bf16x2(pe[0], pe[1]);
+                        dk2[e / 2] = pack_bf16x2(de[0], de[1]);
+                    }
+                }
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const uint32_t off = sw128_offset(t, half * 4 + q4);
+                    st_shared_v4(sP + b * C::kPBytes + off, pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+                    st_shared_v4(sDS + b * C::kPBytes + off, dk2[4 * q4], dk2[4 * q4 + 1], dk2[4 * q4 + 2],
+                                 dk2[4 * q4 + 3]);
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                mbar_arrive(smem_u32(&bar_ds_full[b]));
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ dQ drain, dK/dV epilogue
+        const int quad = warp & 3;
+        const int t = quad * 32 + lane;  // head-dim row of dQ^T; key row of dK/dV
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        int u = 0, kv_items = 0;
+        bool ok = true;
+        for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+            const BwdItem it = decode_bwd2<GLOBAL>(p, k);
+            const int key = it.j * kBN + t;
+            const int64_t kv_off = ((static_cast<int64_t>(it.b) * p.T + key) * p.Hkv + it.kvh) * D;
+            if (it.ntiles == 0) {
+                if (key < p.T) {
+                    for (int c = 0; c < D; c += 8) {
+                        *reinterpret_cast<uint4*>(p.dk + kv_off + c) = make_uint4(0, 0, 0, 0);
+                        *reinterpret_cast<uint4*>(p.dv + kv_off + c) = make_uint4(0, 0, 0, 0);
+                    }
+                }
+                continue;
+            }
+            const int n_it = group * it.ntiles;
+            for (int x = 0; x < n_it; ++x, ++u) {
+                const int h = it.kvh * group + x / it.ntiles;
+                const int i = it.i_lo + x % it.ntiles;
+                const int b = u & 1;
+                ok = mbar_wait(smem_u32(&bar_dq_full[b]), (u >> 1) & 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
+                uint32_t v0[32], v1[32];
+                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b, v0);
+                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + 32, v1);
+                tmem_wait_ld();
+                tc_fence_before();
+                mbar_arrive(smem_u32(&bar_dq_empty[b]));
+                // column c of dQ^T is query row c of the tile: rows outside the
+                // tile's valid range carry exact zeros (dS = 0 there) and land in
+                // padded or neighbouring accumulator rows
+                float* base;
+                if (GLOBAL) base = p.dq_acc + static_cast<int64_t>(i * BQ) * p.Hq * D + h * D + t;
+                else base = p.dq_acc + (static_cast<int64_t>(it.b) * p.T + i * BQ) * p.Hq * D + h * D + t;
+                const int64_t rs = static_cast<int64_t>(p.Hq) * D;
+#pragma unroll
+                for (int c = 0; c < 32; ++c) atomicAdd(base + c * rs, __uint_as_float(v0[c]) * p.scale);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) atomicAdd(base + (32 + c) * rs, __uint_as_float(v1[c]) * p.scale);
+            }
+            if (!ok) break;
+            ok = mbar_wait(smem_u32(&bar_dkv_full), kv_items & 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            tc_fence_after();
+#pragma unroll
+            for (int which = 0; which < 2; ++which) {
+                const uint32_t col = which == 0 ? C::kColDK : C::kColDV;
+                const float mul = which == 0 ? p.scale : 1.0f;
+                logo_bf16* dst = (which == 0 ? p.dk : p.dv) + kv_off;
+#pragma unroll
+                for (int cc = 0; cc < D / 32; ++cc) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + lane_off + col + cc * 32, v);
+                    tmem_wait_ld();
+                    if (key < p.T) {
+#pragma unroll
+                        for (int q4 = 0; q4 < 4; ++q4) {
+                            uint4 w;
+                            w.x = pack_bf16x2(__uint_as_float(v[8 * q4 + 0]) * mul, __uint_as_float(v[8 * q4 + 1]) * mul);
+                            w.y = pack_bf16x2(__uint_as_float(v[8 * q4 + 2]) * mul, __uint_as_float(v[8 * q4 + 3]) * mul);
+                            w.z = pack_bf16x2(__uint_as_float(v[8 * q4 + 4]) * mul, __uint_as_float(v[8 * q4 + 5]) * mul);
+                            w.w = pack_bf16x2(__uint_as_float(v[8 * q4 + 6]) * mul, __uint_as_float(v[8 * q4 + 7]) * mul);
+                            *reinterpret_cast<uint4*>(dst + cc * 32 + q4 * 8) = w;
+                        }
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(smem_u32(&bar_dkv_empty));
+            ++kv_items;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
 // ---------------------------------------------------------------- pre / post
 // Per (row, head): Dsum = sum_d dO * O (fp32); zero the dQ accumulator rows.
 // Global branch: also copy dO_c into the workspace, zero-padding the 128 rows
@@ -524,7 +959,7 @@ size_t local_bwd_ws_layout(const logo_dims& d, char* base, BwdWs* ws)
     const size_t o_ds = off;
     off = round_up(off + rows * d.Hq * sizeof(float), 256);
     const size_t o_dq = off;
-    off = round_up(off + rows * d.Hq * d.D * sizeof(float), 256);
+    off = round_up(off + (rows + kBM) * d.Hq * d.D * sizeof(float), 256);
     if (ws) {
         ws->qc = ws->doc = nullptr;
         ws->dsum = reinterpret_cast<float*>(base + o_ds);
@@ -558,15 +993,23 @@ size_t global_bwd_ws_layout(const logo_dims& d, char* base, BwdWs* ws)
 template <int D, bool GLOBAL>
 int launch_bwd(const BwdParams& prm, cudaStream_t st)
 {
-    using C = BwdCfg<D>;
     static bool attr_done = false;  // benign race: setting the attribute twice is harmless
-    if (!attr_done) {
-        if (set_smem_limit(attn_bwd_kernel<D, GLOBAL>, C::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
-        attr_done = true;
-    }
     const int n_items = prm.B * prm.nblk * prm.Hkv;
     const int grid = max(1, min(n_items, device_sm_count()));
-    attn_bwd_kernel<D, GLOBAL><<<grid, 192, C::kSmemBytes, st>>>(prm);
+    if (D == 128) {
+        if (!attr_done) {
+            if (set_smem_limit(attn_bwd2_kernel<GLOBAL>, Bwd2Cfg::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+            attr_done = true;
+        }
+        attn_bwd2_kernel<GLOBAL><<<grid, Bwd2Cfg::kThreads, Bwd2Cfg::kSmemBytes, st>>>(prm);
+    } else {
+        using C = BwdCfg<D>;
+        if (!attr_done) {
+            if (set_smem_limit(attn_bwd_kernel<D, GLOBAL>, C::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+            attr_done = true;
+        }
+        attn_bwd_kernel<D, GLOBAL><<<grid, 192, C::kSmemBytes, st>>>(prm);
+    }
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
@@ -615,8 +1058,9 @@ extern "C" int logo_local_attn_bwd(const logo_bf16* q, const logo_bf16* k, const
     bwd_pre_kernel<false><<<pre_grid, 128, 0, st>>>(o, dO, nullptr, rows, dims.T, dims.Hq, dims.D, 0, ws.dsum,
                                                     nullptr, ws.dq_acc);
     BwdParams prm{};
-    if (!encode_bf16_4d(&prm.tm_q, q, dims.D, dims.Hq, dims.T, dims.B, 64, kBM) ||
-        !encode_bf16_4d(&prm.tm_do, dO, dims.D, dims.Hq, dims.T, dims.B, 64, kBM) ||
+    const uint32_t qrows = dims.D == 128 ? Bwd2Cfg::kBQ : kBM;
+    if (!encode_bf16_4d(&prm.tm_q, q, dims.D, dims.Hq, dims.T, dims.B, 64, qrows) ||
+        !encode_bf16_4d(&prm.tm_do, dO, dims.D, dims.Hq, dims.T, dims.B, 64, qrows) ||
         !encode_bf16_4d(&prm.tm_k, k, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN) ||
         !encode_bf16_4d(&prm.tm_v, v, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN))
         return LOGO_ERR_CUDA;
@@ -673,8 +1117,9 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
                                                     ws.doc, ws.dq_acc);
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     BwdParams prm{};
-    if (!encode_bf16_4d(&prm.tm_q, ws.qc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, kBM) ||
-        !encode_bf16_4d(&prm.tm_do, ws.doc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, kBM) ||
+    const uint32_t qrows = dims.D == 128 ? Bwd2Cfg::kBQ : kBM;
+    if (!encode_bf16_4d(&prm.tm_q, ws.qc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, qrows) ||
+        !encode_bf16_4d(&prm.tm_do, ws.doc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, qrows) ||
         !encode_bf16_4d(&prm.tm_k, k, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN) ||
         !encode_bf16_4d(&prm.tm_v, v, dims.D, dims.Hkv, dims.T, dims.B, 64, kBN))
         return LOGO_ERR_CUDA;
