@@ -8,11 +8,14 @@
 //   warp 0      TMA producer: Q tile once per item, then K/V blocks through a
 //               ring of shared-memory stages (128-byte swizzle).
 //   warp 1      MMA issuer (one thread): S = Q K^T into one of two TMEM S
-//               buffers, then O += P V into the TMEM O accumulator.
+//               buffers, then O += P V into the TMEM O accumulator with P
+//               read straight from TMEM.
 //   warps 2..5  softmax: one thread per query row (its TMEM lane).  Online
 //               softmax in the log2 domain with conditional rescaling of O
-//               (only when the running max grows by more than 2^8); P is
-//               written to shared memory as bf16 for the P.V MMA.
+//               (only when the running max grows by more than 2^8); P goes
+//               back to TMEM as bf16 pairs, into one of two P buffers, so the
+//               softmax of block n never waits for the P.V of block n-1
+//               unless it has to rescale O.
 // The KV blocks of an item are only those some row can see; blocks where
 // every row sees every key skip the per-element predicate (App. B's
 // three-region traversal; for the local branch the window edge is a second
@@ -32,18 +35,18 @@ namespace {
 
 template <int D>
 struct FwdCfg {
-    static constexpr int kSub = D / 64;                 // 64-column (128-byte) sub-tiles per row
-    static constexpr int kTileBytes = kBM * D * 2;      // one Q / K / V tile
-    static constexpr int kStages = (D == 128) ? 2 : 3;  // K/V ring depth
-    static constexpr int kPBytes = kBM * kBN * 2;
+    static constexpr int kSub = D / 64;             // 64-column (128-byte) sub-tiles per row
+    static constexpr int kTileBytes = kBM * D * 2;  // one Q / K / V tile
+    static constexpr int kStages = 3;               // K/V ring depth
     static constexpr int kOffQ = 0;
     static constexpr int kOffK = kOffQ + kTileBytes;
     static constexpr int kOffV = kOffK + kStages * kTileBytes;
-    static constexpr int kOffP = kOffV + kStages * kTileBytes;
-    static constexpr int kSmemBytes = kOffP + kPBytes + 1024;  // + alignment slack
-    static constexpr uint32_t kColO = 0;
-    static constexpr uint32_t kColS0 = 128;
+    static constexpr int kSmemBytes = kOffV + kStages * kTileBytes + 1024;  // + alignment slack
+    static constexpr uint32_t kColO = 0;     // O accumulator (D columns, fp32)
+    static constexpr uint32_t kColS0 = 128;  // S buffers (128 columns, fp32)
     static constexpr uint32_t kColS1 = 256;
+    static constexpr uint32_t kColP0 = 384;  // P buffers (128 keys as bf16 pairs: 64 columns)
+    static constexpr uint32_t kColP1 = 448;
     static constexpr uint32_t kTmemCols = 512;
 };
 
@@ -96,9 +99,9 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
     using C = FwdCfg<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_p_full, bar_o_done, bar_drain;
+    __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_drain;
     __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_v_full[C::kStages], bar_kv_empty[C::kStages];
-    __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2];
+    __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2], bar_p_full[2], bar_p_free[2];
     __shared__ uint32_t tmem_base_sh;
     __shared__ volatile int abort_flag;
 
@@ -106,14 +109,11 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
     const uint32_t sQ = smem_u32(smem + C::kOffQ);
     const uint32_t sK = smem_u32(smem + C::kOffK);
     const uint32_t sV = smem_u32(smem + C::kOffV);
-    const uint32_t sP = smem_u32(smem + C::kOffP);
 
     if (threadIdx.x == 0) {
         abort_flag = 0;
         mbar_init(smem_u32(&bar_q_full), 1);
         mbar_init(smem_u32(&bar_q_empty), 1);
-        mbar_init(smem_u32(&bar_p_full), 128);
-        mbar_init(smem_u32(&bar_o_done), 1);
         mbar_init(smem_u32(&bar_drain), 1);
         for (int s = 0; s < C::kStages; ++s) {
             mbar_init(smem_u32(&bar_k_full[s]), 1);
@@ -123,6 +123,8 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_s_full[s]), 1);
             mbar_init(smem_u32(&bar_s_empty[s]), 128);
+            mbar_init(smem_u32(&bar_p_full[s]), 128);
+            mbar_init(smem_u32(&bar_p_free[s]), 1);
         }
         fence_mbar_init();
     }
@@ -191,17 +193,18 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
             auto issue_pv = [&](int jj) -> bool {
                 const int itg = s_it + jj;
                 const int st = (kv_it + jj) % C::kStages, f = (kv_it + jj) / C::kStages;
-                if (!mbar_wait(smem_u32(&bar_p_full), itg & 1, &abort_flag)) return false;
+                // per-buffer: the next arrival on this buffer needs this P.V done
+                if (!mbar_wait(smem_u32(&bar_p_full[itg & 1]), (itg >> 1) & 1, &abort_flag)) return false;
                 if (!mbar_wait(smem_u32(&bar_v_full[st]), f & 1, &abort_flag)) return false;
                 tc_fence_after();
                 const uint32_t vbase = sV + st * C::kTileBytes;
+                const uint32_t pcol = tmem + ((itg & 1) ? C::kColP1 : C::kColP0);
 #pragma unroll
                 for (int ks = 0; ks < kBN / 16; ++ks) {
-                    const uint64_t a = sdesc_sw128(sP + (ks >> 2) * 16384 + (ks & 3) * 32, 16, 1024);
                     const uint64_t b = sdesc_sw128(vbase + ks * 2048, 16384, 1024);
-                    umma_bf16_ss(tmem + C::kColO, a, b, idPV, (jj > 0 || ks > 0) ? 1u : 0u);
+                    umma_bf16_ts(tmem + C::kColO, pcol + ks * 8, b, idPV, (jj > 0 || ks > 0) ? 1u : 0u);
                 }
-                umma_commit(smem_u32(&bar_o_done));
+                umma_commit(smem_u32(&bar_p_free[itg & 1]));
                 umma_commit(smem_u32(&bar_kv_empty[st]));
                 return true;
             };
@@ -296,17 +299,17 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                     rs += s[c];
                 }
                 l = l * alpha + rs;
-                // PV of the previous block must be done before O is rescaled
-                // or the P buffer is overwritten.
-                if (itg > 0) {
-                    ok = mbar_wait(smem_u32(&bar_o_done), (itg - 1) & 1, &abort_flag);
+                // O may only be rescaled once the P.V of the previous block is done
+                const bool warp_rescale = __any_sync(0xffffffffu, rescale && n > it.blk_lo);
+                if (warp_rescale) {
+                    // P.V of block itg-1 done: the completion on its P buffer
+                    // (unambiguous: the one before it was awaited a block ago)
+                    ok = mbar_wait(smem_u32(&bar_p_free[(itg - 1) & 1]), ((itg - 1) >> 1) & 1, &abort_flag);
                     __syncwarp();
                     if (!ok) break;
                     tc_fence_after();
-                }
-                // tcgen05.ld/st are warp-collective: rescale if any row of the
-                // warp needs it (the others multiply by alpha = 1).
-                if (__any_sync(0xffffffffu, rescale && n > it.blk_lo)) {
+                    // tcgen05.ld/st are warp-collective: rows that keep their max
+                    // multiply by alpha = 1
                     const uint32_t ocol = tmem + lane_off + C::kColO;
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
@@ -317,21 +320,27 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                         for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
                         tmem_st32(ocol + c * 32, v);
                     }
-                    tmem_wait_st();
                 }
+                // P buffer itg%2 is free once the P.V two blocks back is done
+                ok = mbar_wait(smem_u32(&bar_p_free[itg & 1]), ((itg >> 1) & 1) ^ 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t pcol = tmem + lane_off + ((itg & 1) ? C::kColP1 : C::kColP0);
 #pragma unroll
-                for (int cc = 0; cc < kBN / 8; ++cc) {
-                    const uint32_t addr = sP + (cc >> 3) * 16384 + sw128_offset(r, cc & 7);
-                    st_shared_v4(addr, pack_bf16x2(s[8 * cc + 0], s[8 * cc + 1]), pack_bf16x2(s[8 * cc + 2], s[8 * cc + 3]),
-                                 pack_bf16x2(s[8 * cc + 4], s[8 * cc + 5]), pack_bf16x2(s[8 * cc + 6], s[8 * cc + 7]));
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t pk[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) pk[i] = pack_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
+                    tmem_st32(pcol + 32 * h, pk);
                 }
-                fence_proxy_async_smem();
+                tmem_wait_st();
                 tc_fence_before();
-                mbar_arrive(smem_u32(&bar_p_full));
+                mbar_arrive(smem_u32(&bar_p_full[itg & 1]));
             }
             if (!ok) break;
-            // ---- epilogue: O / l, lse = (m + log2 l) * ln 2
-            ok = mbar_wait(smem_u32(&bar_o_done), (itg - 1) & 1, &abort_flag);
+            // ---- epilogue: O / l, lse = (m + log2 l) * ln 2, once the last P.V is done
+            ok = mbar_wait(smem_u32(&bar_p_free[(itg - 1) & 1]), ((itg - 1) >> 1) & 1, &abort_flag);
             __syncwarp();
             if (!ok) break;
             tc_fence_after();
