@@ -507,7 +507,8 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
     __shared__ uint32_t tmem_base_sh;
     __shared__ volatile int abort_flag;
     __shared__ int sh_pos[2][BQ];
-    __shared__ float2 sh_ld[2][BQ];     // (lse in log2 units, Dsum) per query column
+    // per pair of query columns (2c, 2c+1): (-lse_2c, -lse_2c+1, -Dsum_2c, -Dsum_2c+1), lse in log2 units
+    __shared__ float4 sh_pair[2][BQ / 2];
     __shared__ int sh_open[2][2];       // per staging warp: every column sees every key of the block
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -679,39 +680,51 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             const int k0 = it.j * kBN;
             const int key = k0 + t;
             const int n_it = group * it.ntiles;
-            for (int x = 0; x < n_it; ++x, ++u) {
+            // staging values of tile x (query positions, lse in log2 units,
+            // Dsum, "sees every key" flag): loaded one tile ahead so the global
+            // loads overlap the previous tile's work
+            int pf_pos = -1;
+            float2 pf_ld = make_float2(0.f, 0.f);
+            bool pf_open = false;
+            auto load_stage = [&](int x) {
                 const int h = it.kvh * group + x / it.ntiles;
                 const int i = it.i_lo + x % it.ntiles;
-                const int b = u & 1;
-                if (tw < BQ) {  // stage the tile's query positions, lse (log2 units), Dsum
-                    int pc = -1;
-                    float2 ld = make_float2(0.f, 0.f);
-                    bool open = false;  // this column sees every key of the block
-                    if (!GLOBAL) {
-                        const int q = i * BQ + tw;
-                        if (q < p.T) {
-                            const int64_t idx = (static_cast<int64_t>(it.b) * p.Hq + h) * p.T + q;
-                            pc = q;
-                            ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
-                            open = q >= k0 + kBN - 1 && q - k0 < window;
-                        }
-                    } else {
-                        const int row = i * BQ + tw;
-                        if (row >= it.row_lo && row < it.row_hi) {
-                            const int64_t idx = static_cast<int64_t>(h) * p.cap + row;
-                            pc = p.pos[row];
-                            ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
-                            open = pc >= k0 + kBN - 1;
-                        }
+                pf_pos = -1;
+                pf_ld = make_float2(0.f, 0.f);
+                pf_open = false;
+                if (!GLOBAL) {
+                    const int q = i * BQ + tw;
+                    if (q < p.T) {
+                        const int64_t idx = (static_cast<int64_t>(it.b) * p.Hq + h) * p.T + q;
+                        pf_pos = q;
+                        pf_ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
+                        pf_open = q >= k0 + kBN - 1 && q - k0 < window;
                     }
-                    sh_pos[b][tw] = pc;
-                    sh_ld[b][tw] = ld;
-                    const bool all_open = __all_sync(0xffffffffu, open);
+                } else {
+                    const int row = i * BQ + tw;
+                    if (row >= it.row_lo && row < it.row_hi) {
+                        const int64_t idx = static_cast<int64_t>(h) * p.cap + row;
+                        pf_pos = p.pos[row];
+                        pf_ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
+                        pf_open = pf_pos >= k0 + kBN - 1;
+                    }
+                }
+            };
+            if (tw < BQ) load_stage(0);
+            for (int x = 0; x < n_it; ++x, ++u) {
+                const int b = u & 1;
+                if (tw < BQ) {
+                    sh_pos[b][tw] = pf_pos;
+                    float* pr = reinterpret_cast<float*>(&sh_pair[b][tw >> 1]);
+                    pr[tw & 1] = -pf_ld.x;
+                    pr[2 + (tw & 1)] = -pf_ld.y;
+                    const bool all_open = __all_sync(0xffffffffu, pf_open);
                     if (lane == 0) sh_open[b][tw >> 5] = all_open ? 1 : 0;
                 }
                 mbar_arrive(smem_u32(&bar_stage));
                 ok = mbar_wait(smem_u32(&bar_stage), u & 1, &abort_flag);
                 if (!ok) break;
+                if (tw < BQ && x + 1 < n_it) load_stage(x + 1);
                 const bool open = sh_open[b][0] && sh_open[b][1];
                 ok = mbar_wait(smem_u32(&bar_st_full[b]), (u >> 1) & 1, &abort_flag);
                 __syncwarp();
@@ -727,37 +740,29 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + 64 + half * 32, dpv);
                 tmem_wait_ld();
                 uint32_t pk[16], dk2[16];
-                if (open) {
+                // P = 2^(S*scale*log2e - lse), dS = P (dP - Dsum), two columns per
+                // f32x2 instruction; masked tiles also test each column's position
+                const uint64_t scale2 = f2_pack(p.scale_log2, p.scale_log2);
 #pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        float pe[2], de[2];
-#pragma unroll
-                        for (int zz = 0; zz < 2; ++zz) {
-                            const float2 ld = sh_ld[b][half * 32 + e + zz];
-                            const float pr = ex2_approx(fmaf(__uint_as_float(sv[e + zz]), p.scale_log2, -ld.x));
-                            pe[zz] = pr;
-                            de[zz] = pr * (__uint_as_float(dpv[e + zz]) - ld.y);
-                        }
-                        pk[e / 2] = pack_bf16x2(pe[0], pe[1]);
-                        dk2[e / 2] = pack_bf16x2(de[0], de[1]);
+                for (int e = 0; e < 32; e += 2) {
+                    const int c = half * 32 + e;
+                    const float4 q = sh_pair[b][c >> 1];
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), scale2,
+                                     f2_pack(q.x, q.y)),
+                              x0, x1);
+                    float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                    if (!open) {
+                        if (!key_visible(key, sh_pos[b][c], window)) p0 = 0.f;
+                        if (!key_visible(key, sh_pos[b][c + 1], window)) p1 = 0.f;
                     }
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        float pe[2], de[2];
-#pragma unroll
-                        for (int zz = 0; zz < 2; ++zz) {
-                            const int c = half * 32 + e + zz;
-                            const float2 ld = sh_ld[b][c];
-                            const bool vis = key_visible(key, sh_pos[b][c], window);
-                            const float pr =
-                                vis ? ex2_approx(fmaf(__uint_as_float(sv[e + zz]), p.scale_log2, -ld.x)) : 0.f;
-                            pe[zz] = pr;
-                            de[zz] = pr * (__uint_as_float(dpv[e + zz]) - ld.y);
-                        }
-                        pk[e / 2] = pack_bf16x2(pe[0], pe[1]);
-                        dk2[e / 2] = pack_bf16x2(de[0], de[1]);
-                    }
+                    const uint64_t pp = f2_pack(p0, p1);
+                    const uint64_t t2 =
+                        f2_add(f2_pack(__uint_as_float(dpv[e]), __uint_as_float(dpv[e + 1])), f2_pack(q.z, q.w));
+                    float d0, d1;
+                    f2_unpack(f2_mul(pp, t2), d0, d1);
+                    pk[e / 2] = cvt_bf16x2(p0, p1);
+                    dk2[e / 2] = cvt_bf16x2(d0, d1);
                 }
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {

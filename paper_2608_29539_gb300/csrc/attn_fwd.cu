@@ -265,13 +265,15 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                 tc_fence_after();
                 float s[kBN];
                 const uint32_t scol = tmem + lane_off + (buf ? C::kColS1 : C::kColS0);
+                {
+                    uint32_t v[kBN / 32][32];
 #pragma unroll
-                for (int c = 0; c < kBN / 32; ++c) {
-                    uint32_t v[32];
-                    tmem_ld32(scol + c * 32, v);
-                    tmem_wait_ld();
+                    for (int c = 0; c < kBN / 32; ++c) tmem_ld32(scol + c * 32, v[c]);
+                    tmem_wait_ld();  // one wait for all four loads
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[i]);
+                    for (int c = 0; c < kBN / 32; ++c)
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[c][i]);
                 }
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_s_empty[buf]));
@@ -280,9 +282,20 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                     for (int c = 0; c < kBN; ++c)
                         if (!key_visible(n * kBN + c, mypos, window)) s[c] = -INFINITY;
                 }
-                float mx = -INFINITY;
+                // 4 independent 3-input max chains and 4 packed-pair sums keep
+                // dependency chains short; exp arguments are formed two at a
+                // time with f32x2 FMAs
+                float mx4[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
-                for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
+                for (int c = 4; c < kBN; c += 8) {
+                    mx4[0] = max3f(mx4[0], s[c], s[c + 1]);
+                    mx4[1] = max3f(mx4[1], s[c + 2], s[c + 3]);
+                    if (c + 4 < kBN) {
+                        mx4[2] = max3f(mx4[2], s[c + 4], s[c + 5]);
+                        mx4[3] = max3f(mx4[3], s[c + 6], s[c + 7]);
+                    }
+                }
+                const float mx = max3f(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
                 const float m_new = fmaxf(m_ref, mx * p.scale_log2);
                 float alpha = 1.f;
                 bool rescale = false;
@@ -292,11 +305,25 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                     rescale = true;
                 }
                 const float m_use = (m_ref == -INFINITY) ? 0.f : m_ref;
-                float rs = 0.f;
+                const uint64_t scale2 = f2_pack(p.scale_log2, p.scale_log2);
+                const uint64_t negm2 = f2_pack(-m_use, -m_use);
+                uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-                for (int c = 0; c < kBN; ++c) {
-                    s[c] = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
-                    rs += s[c];
+                for (int c = 0; c < kBN; c += 2) {
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(s[c], s[c + 1]), scale2, negm2), x0, x1);
+                    s[c] = ex2_approx(x0);
+                    s[c + 1] = ex2_approx(x1);
+                    acc2[(c >> 1) & 3] = f2_add(acc2[(c >> 1) & 3], f2_pack(s[c], s[c + 1]));
+                }
+                float rs;
+                {
+                    float a0, a1, b0, b1, c0, c1, d0, d1;
+                    f2_unpack(acc2[0], a0, a1);
+                    f2_unpack(acc2[1], b0, b1);
+                    f2_unpack(acc2[2], c0, c1);
+                    f2_unpack(acc2[3], d0, d1);
+                    rs = ((a0 + a1) + (b0 + b1)) + ((c0 + c1) + (d0 + d1));
                 }
                 l = l * alpha + rs;
                 // O may only be rescaled once the P.V of the previous block is done
@@ -331,7 +358,7 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                 for (int h = 0; h < 2; ++h) {
                     uint32_t pk[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) pk[i] = pack_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
+                    for (int i = 0; i < 32; ++i) pk[i] = cvt_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
                     tmem_st32(pcol + 32 * h, pk);
                 }
                 tmem_wait_st();
