@@ -52,7 +52,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
-    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="16k (headline), 4k, 64k, or sweep:<ratio> (T=32K, H=16, W=1024)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -268,13 +269,20 @@ def oracle_sample(w, x, budget_s, pos_by_seq):
 
 
 # ------------------------------------------------------------------ arms
+def workload_named(name):
+    from paper_2608_29539_gb300.workloads import WORKLOADS, sweep
+    if name.startswith("sweep:"):
+        return sweep(float(name.split(":", 1)[1]))
+    return WORKLOADS[name]
+
+
 def reference_arm(a, rank, world):
     """The oracle, as it stands, on the host cores: same metric and config."""
     if rank != 0:
         return
-    from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
+    from paper_2608_29539_gb300.workloads import make_inputs
     import oracle
-    w = WORKLOADS[a.workload]
+    w = workload_named(a.workload)
     x = make_inputs(w, device="cpu")
     p = x["p"].numpy()
     z = oracle.select_ratio(p, w.k_per_seq) if w.mode == "ratio" else oracle.select_threshold(p, x["b_th"])
@@ -308,8 +316,7 @@ def config_of(w):
 
 def native_arm(a, rank, world, local_rank, dist_on):
     from paper_2608_29539_gb300 import logo as L
-    from paper_2608_29539_gb300.workloads import WORKLOADS
-    w = WORKLOADS[a.workload]
+    w = workload_named(a.workload)
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     pk = peaks()
@@ -354,6 +361,7 @@ def native_arm(a, rank, world, local_rank, dist_on):
     # roofline of the dominant call (its tensor-core kernel dominates the call)
     flops_call = {"local_fwd": fl_local * 4 / 14, "local_bwd": fl_local * 10 / 14,
                   "global_fwd": fl_global * 4 / 14, "global_bwd": fl_global * 10 / 14}
+    g_ms = per_call["global_fwd"] + per_call["global_bwd"]
     dom = max(flops_call, key=lambda c: per_call[c])
     achieved = flops_call[dom] / (per_call[dom] / 1e3) / 1e12
     kernel_src = os.path.join(ROOT, "paper_2608_29539_gb300", "csrc",
@@ -363,7 +371,6 @@ def native_arm(a, rank, world, local_rank, dist_on):
             "frac": achieved / pk["bf16_sus"], "traffic": tr,
             "peak_note": f"{pk['src']} sustained bf16 (kernel timed inside a multi-ms step); "
                          f"frac of burst peak {achieved / pk['bf16']:.3f}"}
-    g_ms = per_call["global_fwd"] + per_call["global_bwd"]
     l_ms = per_call["local_fwd"] + per_call["local_bwd"]
     breakdown = {c: {"ms": per_call[c]} for c in CALLS}
     for c, fl in flops_call.items():
@@ -394,7 +401,7 @@ def native_arm(a, rank, world, local_rank, dist_on):
         dense_ms = float(np.median(tt))
         dense_flops = w.B * w.T * (w.T + 1) // 2 * 14 * w.D * w.Hq
         line["dense_global_fwd_bwd"] = {"ms": dense_ms, "tflops": dense_flops / (dense_ms / 1e3) / 1e12,
-                                        "speedup_sparse_vs_dense": dense_ms / g_ms,
+                                        "speedup_sparse_vs_dense": dense_ms / max(g_ms, 1e-9),
                                         "ideal_speedup": dense_flops / max(fl_global, 1)}
         del dl
 

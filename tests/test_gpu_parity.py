@@ -359,3 +359,66 @@ def test_full_size_16k_workload_sampled():
     check_close(np32(layer.dqG)[:, :, h], dense[:, :, h], "dqG head 7")
     check_close(np32(layer.dkG)[:, :, h], rdk[:, :, h], "dkG head 7")
     check_close(np32(layer.dvG)[:, :, h], rdv[:, :, h], "dvG head 7")
+
+
+def test_full_size_64k_gqa_sampled():
+    """The 64K GQA workload (B=1, Hq=32, Hkv=8, d=128, T=65536, W=2048, ratio
+    1/16) through the benchmark's layer object.  Selection in full; forward
+    rows sampled; combine on a token subset; dQ on sampled rows (a row's dQ
+    depends only on its own keys); dK/dV on a 64-key range, computed by the
+    oracle from every query row that can see those keys (so they are
+    complete), for one KV head (its whole query group)."""
+    import bench
+    from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
+    w = WORKLOADS["64k"]
+    x = make_inputs(w, device="cuda")
+    layer = bench.layer_for(w, torch.device("cuda"))
+    bench.run_step(layer, x)
+    torch.cuda.synchronize()
+    assert L().logo_get_device_status() == 0
+    n = int(layer.n_sel.item())
+    oz, opos, ocu, orow, on = oracle_select(x["p"].cpu(), 1, 0.0, w.ratio)
+    assert n == on == w.k_per_seq
+    np.testing.assert_array_equal(layer.pos[:n].cpu().numpy(), opos)
+    np.testing.assert_array_equal(layer.row_of.cpu().numpy(), orow)
+    f = lambda k: np32(x[k])  # noqa: E731
+    qL, kL, vL, qG, kG, vG = (f(k) for k in ("qL", "kL", "vL", "qG", "kG", "vG"))
+    rng = np.random.default_rng(1)
+    heads = [0, 5, 31]
+    rows = np.sort(np.concatenate([rng.choice(w.T, 96, replace=False), [0, 2047, 2048, w.T - 1]])).astype(np.int32)
+    ro, _ = oracle.attn_fwd(qL, kL, vL, np.zeros_like(rows), rows, w.window, heads=heads)
+    check_close(np32(layer.o_l)[0, rows][:, heads], ro[:, heads], "o_l sampled")
+    grow = np.sort(np.concatenate([rng.choice(n, 96, replace=False), [0, n - 1]]))
+    rog, _ = oracle.attn_fwd(qG, kG, vG, np.zeros(len(grow), np.int32), opos[grow], 0, heads=heads)
+    check_close(np32(layer.o_c)[grow][:, heads], rog[:, heads], "o_c sampled")
+    # combine on the first 4096 tokens (their selected rows re-packed)
+    tt = 4096
+    z_sub = oz[:, :tt]
+    sel_rows = orow[0, :tt][z_sub[0] == 1]
+    row_sub = -np.ones((1, tt), np.int32)
+    row_sub[0, z_sub[0] == 1] = np.arange(len(sel_rows), dtype=np.int32)
+    o_l = np32(layer.o_l)[:, :tt]
+    rfo, _, _ = oracle.combine_fwd(o_l, np32(layer.o_c)[sel_rows], f("p")[:, :tt], z_sub, row_sub)
+    check_close(np32(layer.o)[:, :tt], rfo, "o (first 4096 tokens)")
+    group = w.Hq // w.Hkv
+    kvh = 2
+    hs = list(range(kvh * group, (kvh + 1) * group))
+    dOL = np32(layer.dO_l)[0]
+    # local: dq on sampled rows; dK/dV on keys [s0, s0+64) from every row that sees them
+    s0 = 20000
+    lrows = np.arange(s0, s0 + 64 + w.window - 1, dtype=np.int32)
+    rdq, rdk, rdv = oracle.attn_bwd(qL, kL, vL, np.zeros_like(lrows), lrows, w.window, dOL[lrows], heads=hs)
+    check_close(np32(layer.dkL)[0, s0:s0 + 64, kvh], rdk[0, s0:s0 + 64, kvh], "dkL key range")
+    check_close(np32(layer.dvL)[0, s0:s0 + 64, kvh], rdv[0, s0:s0 + 64, kvh], "dvL key range")
+    check_close(np32(layer.dqL)[0, lrows][:, hs], rdq[:, hs], "dqL rows")
+    # global: keys near the end so that few selected rows see them
+    s1 = w.T - 1024
+    grows = np.nonzero(opos >= s1)[0]
+    dOc = np32(layer.dO_c)[:n]
+    rdq, rdk, rdv = oracle.attn_bwd(qG, kG, vG, np.zeros(len(grows), np.int32), opos[grows], 0, dOc[grows], heads=hs)
+    check_close(np32(layer.dkG)[0, s1:s1 + 64, kvh], rdk[0, s1:s1 + 64, kvh], "dkG key range")
+    check_close(np32(layer.dvG)[0, s1:s1 + 64, kvh], rdv[0, s1:s1 + 64, kvh], "dvG key range")
+    check_close(np32(layer.dqG)[0, opos[grows]][:, hs], rdq[:, hs], "dqG rows")
+    # unselected rows of the dense global dQ are exactly zero
+    unsel = np.setdiff1d(np.arange(w.T), opos)[:4096]
+    assert not np32(layer.dqG)[0, unsel].any()
