@@ -59,6 +59,7 @@ struct FwdParams {
     const int32_t* pos;            // global: packed positions
     const GlobalTile* tiles;       // global: schedule
     const int32_t* n_tiles;        // global: schedule length (device)
+    int32_t* next_item;            // global: work counter, zeroed by the schedule kernel
     int B, T, Hq, Hkv, window, cap;
     int q_tiles;                   // local: query tiles per sequence
     float scale_log2;              // softmax scale * log2(e)
@@ -104,6 +105,11 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
     __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2], bar_p_full[2], bar_p_free[2];
     __shared__ uint32_t tmem_base_sh;
     __shared__ volatile int abort_flag;
+    // global branch: items are taken dynamically (longest first, whichever CTA
+    // is free next); the producer passes each index to the other roles
+    // through this 4-slot ring (-1 ends the work)
+    __shared__ volatile int item_ring[4];
+    __shared__ __align__(8) uint64_t bar_item_full[4], bar_item_empty[4];
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t sQ = smem_u32(smem + C::kOffQ);
@@ -119,6 +125,10 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
             mbar_init(smem_u32(&bar_k_full[s]), 1);
             mbar_init(smem_u32(&bar_v_full[s]), 1);
             mbar_init(smem_u32(&bar_kv_empty[s]), 1);
+        }
+        for (int s = 0; s < 4; ++s) {
+            mbar_init(smem_u32(&bar_item_full[s]), 1);
+            mbar_init(smem_u32(&bar_item_empty[s]), 5);  // the MMA thread + one lane per softmax warp
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_s_full[s]), 1);
@@ -138,6 +148,26 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
 
+    // u-th work item of this CTA for a consumer role, or -1 when done.
+    // whole_warp: called by all 32 lanes (the softmax warps), which then
+    // arrive once per warp; otherwise by the single MMA-issuing thread.
+    auto consume_item = [&](int u, bool* ok, bool whole_warp) -> int {
+        if (!GLOBAL) {
+            const int k = blockIdx.x + u * gridDim.x;
+            return k < n_items ? k : -1;
+        }
+        const int slot = u & 3;
+        if (!(*ok = mbar_wait(smem_u32(&bar_item_full[slot]), (u >> 2) & 1, &abort_flag))) return -1;
+        const int k = item_ring[slot];
+        if (whole_warp) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bar_item_empty[slot]));
+        } else {
+            mbar_arrive(smem_u32(&bar_item_empty[slot]));
+        }
+        return k;
+    };
+
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
@@ -151,7 +181,20 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
             for (int s = 0; s < C::kStages; ++s) last_fill[s] = -1;
             int q_fills = 0;
             bool ok = true;
-            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x, ++item_i) {
+            for (;; ++item_i) {
+                int k;
+                if (GLOBAL) {
+                    const int slot = item_i & 3;
+                    if (!(ok = mbar_wait(smem_u32(&bar_item_empty[slot]), ((item_i >> 2) & 1) ^ 1, &abort_flag))) break;
+                    k = atomicAdd(p.next_item, 1);
+                    if (k >= n_items) k = -1;
+                    item_ring[slot] = k;
+                    mbar_arrive(smem_u32(&bar_item_full[slot]));
+                } else {
+                    k = blockIdx.x + item_i * gridDim.x;
+                    if (k >= n_items) k = -1;
+                }
+                if (k < 0) break;
                 const FwdItem it = decode_item<GLOBAL>(p, k);
                 if (!(ok = mbar_wait(smem_u32(&bar_q_empty), (item_i & 1) ^ 1, &abort_flag))) break;
                 const uint32_t qb = smem_u32(&bar_q_full);
@@ -173,6 +216,7 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                                     pol_kv);
                     last_fill[st] = f;
                 }
+                if (!ok) break;
             }
             if (!ok) {  // let copies already issued land before the CTA exits
                 if (q_fills > 0) mbar_wait_drain(smem_u32(&bar_q_full), (q_fills - 1) & 1);
@@ -208,7 +252,9 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                 umma_commit(smem_u32(&bar_kv_empty[st]));
                 return true;
             };
-            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x, ++item_i) {
+            for (;; ++item_i) {
+                const int k = consume_item(item_i, &ok, false);
+                if (k < 0) break;
                 const FwdItem it = decode_item<GLOBAL>(p, k);
                 const int nblk = it.blk_hi - it.blk_lo + 1;
                 if (!(ok = mbar_wait(smem_u32(&bar_q_full), item_i & 1, &abort_flag))) break;
@@ -249,7 +295,9 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
         const int window = GLOBAL ? kNoWindow : p.window;
         int itg = 0;
         bool ok = true;
-        for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+        for (int item_i = 0;; ++item_i) {
+            const int k = consume_item(item_i, &ok, true);
+            if (k < 0) break;
             const FwdItem it = decode_item<GLOBAL>(p, k);
             const bool row_valid = r < it.nrows;
             int mypos;
@@ -417,7 +465,8 @@ __global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __
                                                                int32_t* __restrict__ tile_off,
                                                                GlobalTile* __restrict__ unsorted,
                                                                GlobalTile* __restrict__ sorted,
-                                                               int32_t* __restrict__ n_tiles)
+                                                               int32_t* __restrict__ n_tiles,
+                                                               int32_t* __restrict__ next_item)
 {
     __shared__ int sh_nt;
     if (threadIdx.x == 0) {
@@ -429,6 +478,7 @@ __global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __
         tile_off[B] = acc;
         sh_nt = acc;
         *n_tiles = acc;
+        *next_item = 0;
     }
     __syncthreads();
     const int nt = sh_nt;
@@ -468,6 +518,7 @@ struct GlobalFwdWs {
     GlobalTile* sorted;
     int32_t* tile_off;
     int32_t* n_tiles;
+    int32_t* next_item;
 };
 
 size_t global_fwd_ws_layout(const logo_dims& d, char* base, GlobalFwdWs* ws)
@@ -484,13 +535,14 @@ size_t global_fwd_ws_layout(const logo_dims& d, char* base, GlobalFwdWs* ws)
     const size_t o_to = off;
     off = round_up(off + (d.B + 1) * sizeof(int32_t), 256);
     const size_t o_nt = off;
-    off = round_up(off + sizeof(int32_t), 256);
+    off = round_up(off + 2 * sizeof(int32_t), 256);
     if (ws) {
         ws->qc = reinterpret_cast<logo_bf16*>(base + o_qc);
         ws->unsorted = reinterpret_cast<GlobalTile*>(base + o_un);
         ws->sorted = reinterpret_cast<GlobalTile*>(base + o_so);
         ws->tile_off = reinterpret_cast<int32_t*>(base + o_to);
         ws->n_tiles = reinterpret_cast<int32_t*>(base + o_nt);
+        ws->next_item = ws->n_tiles + 1;
     }
     return off;
 }
@@ -582,7 +634,8 @@ extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* 
     const int row_elems = dims.Hq * dims.D;
     const int gather_grid = max(1, min(cap + kBM, device_sm_count() * 8));
     gather_rows_kernel<<<gather_grid, 256, 0, st>>>(q, pos, cu_q, n_sel_total, dims.B, dims.T, row_elems, ws.qc);
-    global_schedule_kernel<<<1, 1024, 0, st>>>(pos, cu_q, dims.B, ws.tile_off, ws.unsorted, ws.sorted, ws.n_tiles);
+    global_schedule_kernel<<<1, 1024, 0, st>>>(pos, cu_q, dims.B, ws.tile_off, ws.unsorted, ws.sorted, ws.n_tiles,
+                                               ws.next_item);
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     FwdParams prm{};
     if (!encode_bf16_4d(&prm.tm_q, ws.qc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, kBM) ||
@@ -594,6 +647,7 @@ extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* 
     prm.pos = pos;
     prm.tiles = ws.sorted;
     prm.n_tiles = ws.n_tiles;
+    prm.next_item = ws.next_item;
     prm.B = dims.B;
     prm.T = dims.T;
     prm.Hq = dims.Hq;
