@@ -43,7 +43,11 @@ L2_BYTES = 129 * 1024 * 1024
 # DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by
 # the SHA-256 of the kernel source it was taken on; reported only while the
 # source is unchanged (see profiles/).
-TRAFFIC = {}
+TRAFFIC = {
+    # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
+    ("local_bwd", "521ac9082c101078"): 821543936 + 479842048,
+    ("global_bwd", "521ac9082c101078"): 428666112 + 294057472,
+}
 
 
 def parse():
@@ -224,7 +228,7 @@ def sum_over_ranks(x, dist_on):
 
 
 # ------------------------------------------------------------------ cpu side
-def oracle_sample(w, x, budget_s, pos_by_seq):
+def oracle_sample(w, x, budget_s, pos_by_seq, rows=None):
     """Time the oracle on a bounded sample of the workload: the first
     `nh` heads, the last `r` query rows of each branch of sequence 0 (the most
     expensive rows), forward + backward.  Returns (useful TFLOP/s, seconds,
@@ -257,15 +261,24 @@ def oracle_sample(w, x, budget_s, pos_by_seq):
         pairs = sum(min(t + 1, w.window) for t in lt.tolist()) + int((gt.astype(np.int64) + 1).sum())
         return dt, pairs * nh * 14 * w.D
 
-    r0 = 8
-    dt0, _ = run(r0, min(r0, len(sel)))
-    scale = max(1.0, budget_s / max(dt0, 1e-3))
-    r = int(min(T, r0 * scale))
-    rg = int(min(len(sel), r0 * scale))
+    if rows is None:
+        # grow the sample (doubling the rows) until one run fills about a
+        # quarter of the budget, then size the final run to the budget
+        r, dt = 8, 0.0
+        while True:
+            dt, _ = run(min(r, T), min(r, len(sel)))
+            if dt >= budget_s / 4 or (r >= T and r >= len(sel)):
+                break
+            r *= 2
+        scale = max(1.0, budget_s / max(dt, 1e-3))
+        r = int(min(T, r * scale))
+        rg = int(min(len(sel), r))
+    else:
+        r, rg = rows
     dt, flops = run(r, rg)
     desc = (f"oracle fp64 fwd+bwd on heads 0..{nh - 1} of sequence 0: the last {r} local query rows and the last "
             f"{rg} selected global rows (the most expensive rows); useful FLOPs counted as on the GPU")
-    return flops / dt / 1e12, dt, nth, desc
+    return flops / dt / 1e12, dt, nth, desc, (r, rg)
 
 
 # ------------------------------------------------------------------ arms
@@ -290,8 +303,9 @@ def reference_arm(a, rank, world):
     pos_by_seq = [pos[cu_q[b]:cu_q[b + 1]] for b in range(w.B)]
     per_step = max(2.0, 150.0 / max(1, a.steps + a.warmup))
     vals, secs = [], []
+    rows = None  # sized once (first warm-up step), then fixed
     for i in range(a.warmup + a.steps):
-        v, dt, nth, desc = oracle_sample(w, x, per_step, pos_by_seq)
+        v, dt, nth, desc, rows = oracle_sample(w, x, per_step, pos_by_seq, rows)
         if i >= a.warmup:
             vals.append(v)
             secs.append(dt)
@@ -441,7 +455,7 @@ def native_arm(a, rank, world, local_rank, dist_on):
     # ---- the oracle on the host cores (rank 0, N = 1 only)
     if rank == 0 and world == 1 and not a.no_cpu_baseline:
         xc = {k: x[k][:1].cpu() for k in ("qL", "kL", "vL", "qG", "kG", "vG")}
-        v, dt, nth, desc = oracle_sample(w, xc, a.cpu_budget, pos_by_seq)
+        v, dt, nth, desc, _ = oracle_sample(w, xc, a.cpu_budget, pos_by_seq)
         line["cpu_baseline"] = {"value": v, "unit": "TFLOP/s", "cores": nth, "kind": "oracle", "sample": desc,
                                 "seconds": dt}
     if rank == 0:
