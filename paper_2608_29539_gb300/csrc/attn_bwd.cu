@@ -65,6 +65,7 @@ struct BwdParams {
     logo_bf16* dv;
     const int32_t* pos;
     const int32_t* cu_q;
+    const int32_t* first_row;  // global: [B, nblk] first packed row of sequence b whose position reaches block j
     int B, T, Hq, Hkv, window, cap, nblk, q_tiles;
     float scale, scale_log2;
 };
@@ -477,12 +478,7 @@ __device__ __forceinline__ BwdItem decode_bwd2(const BwdParams& p, int k)
     } else {
         it.row_lo = p.cu_q[it.b];
         it.row_hi = p.cu_q[it.b + 1];
-        int lo = it.row_lo, hi = it.row_hi;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (p.pos[mid] < k0) lo = mid + 1;
-            else hi = mid;
-        }
+        const int lo = p.first_row[it.b * p.nblk + it.j];  // precomputed search (App. B)
         if (lo >= it.row_hi) {
             it.i_lo = 0;
             it.ntiles = 0;
@@ -916,6 +912,26 @@ __global__ void __launch_bounds__(128) bwd_pre_kernel(const logo_bf16* __restric
     }
 }
 
+// For every sequence b and KV block j: the first packed row of b whose
+// position reaches the block's first key (App. B's precomputed search that
+// lets the backward skip every query tile before it).
+__global__ void __launch_bounds__(256) first_row_kernel(const int32_t* __restrict__ pos,
+                                                        const int32_t* __restrict__ cu_q, int B, int nblk,
+                                                        int32_t* __restrict__ first_row)
+{
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= B * nblk) return;
+    const int b = idx / nblk, j = idx % nblk;
+    int lo = cu_q[b], hi = cu_q[b + 1];
+    const int k0 = j * kBN;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (pos[mid] < k0) lo = mid + 1;
+        else hi = mid;
+    }
+    first_row[idx] = lo;
+}
+
 // dQ accumulator (fp32) -> dq (bf16).  Local: elementwise.  Global: every
 // dense token writes its packed row's gradient, or zeros if not selected.
 template <bool GLOBAL>
@@ -955,6 +971,7 @@ struct BwdWs {
     logo_bf16* doc;
     float* dsum;
     float* dq_acc;
+    int32_t* first_row;
 };
 
 size_t local_bwd_ws_layout(const logo_dims& d, char* base, BwdWs* ws)
@@ -969,6 +986,7 @@ size_t local_bwd_ws_layout(const logo_dims& d, char* base, BwdWs* ws)
         ws->qc = ws->doc = nullptr;
         ws->dsum = reinterpret_cast<float*>(base + o_ds);
         ws->dq_acc = reinterpret_cast<float*>(base + o_dq);
+        ws->first_row = nullptr;
     }
     return off;
 }
@@ -986,7 +1004,10 @@ size_t global_bwd_ws_layout(const logo_dims& d, char* base, BwdWs* ws)
     off = round_up(off + cap * d.Hq * sizeof(float), 256);
     const size_t o_dq = off;
     off = round_up(off + rows * d.Hq * d.D * sizeof(float), 256);
+    const size_t o_fr = off;
+    off = round_up(off + static_cast<size_t>(d.B) * ((d.T + kBN - 1) / kBN) * sizeof(int32_t), 256);
     if (ws) {
+        ws->first_row = reinterpret_cast<int32_t*>(base + o_fr);
         ws->qc = reinterpret_cast<logo_bf16*>(base + o_qc);
         ws->doc = reinterpret_cast<logo_bf16*>(base + o_do);
         ws->dsum = reinterpret_cast<float*>(base + o_ds);
@@ -1120,6 +1141,8 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     gather_rows_kernel<<<grid_rows, 256, 0, st>>>(q, pos, cu_q, n_sel_total, dims.B, dims.T, row_elems, ws.qc);
     bwd_pre_kernel<true><<<grid_rows, 128, 0, st>>>(o_c, dO_c, n_sel_total, 0, dims.T, dims.Hq, dims.D, cap, ws.dsum,
                                                     ws.doc, ws.dq_acc);
+    const int nblk = (dims.T + kBN - 1) / kBN;
+    first_row_kernel<<<(dims.B * nblk + 255) / 256, 256, 0, st>>>(pos, cu_q, dims.B, nblk, ws.first_row);
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     BwdParams prm{};
     const uint32_t qrows = dims.D == 128 ? Bwd2Cfg::kBQ : kBM;
@@ -1135,6 +1158,7 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     prm.dv = dv;
     prm.pos = pos;
     prm.cu_q = cu_q;
+    prm.first_row = ws.first_row;
     prm.B = dims.B;
     prm.T = dims.T;
     prm.Hq = dims.Hq;
