@@ -27,6 +27,7 @@
 #include <cuda_bf16.h>
 
 #include <cstdint>
+#include <type_traits>
 
 #include "attn_common.cuh"
 #include "host_common.h"
@@ -737,29 +738,35 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 tmem_wait_ld();
                 uint32_t pk[16], dk2[16];
                 // P = 2^(S*scale*log2e - lse), dS = P (dP - Dsum), two columns per
-                // f32x2 instruction; masked tiles also test each column's position
+                // f32x2 instruction.  Two branch-free copies of the loop (open
+                // tiles skip the visibility test) so that the iterations overlap.
                 const uint64_t scale2 = f2_pack(p.scale_log2, p.scale_log2);
+                auto columns = [&](auto masked) {
+                    constexpr bool kMasked = decltype(masked)::value;
 #pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    const int c = half * 32 + e;
-                    const float4 q = sh_pair[b][c >> 1];
-                    float x0, x1;
-                    f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), scale2,
-                                     f2_pack(q.x, q.y)),
-                              x0, x1);
-                    float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-                    if (!open) {
-                        if (!key_visible(key, sh_pos[b][c], window)) p0 = 0.f;
-                        if (!key_visible(key, sh_pos[b][c + 1], window)) p1 = 0.f;
+                    for (int e = 0; e < 32; e += 2) {
+                        const int c = half * 32 + e;
+                        const float4 q = sh_pair[b][c >> 1];
+                        float x0, x1;
+                        f2_unpack(f2_fma(f2_pack(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), scale2,
+                                         f2_pack(q.x, q.y)),
+                                  x0, x1);
+                        float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+                        if constexpr (kMasked) {
+                            p0 = key_visible(key, sh_pos[b][c], window) ? p0 : 0.f;
+                            p1 = key_visible(key, sh_pos[b][c + 1], window) ? p1 : 0.f;
+                        }
+                        const uint64_t pp = f2_pack(p0, p1);
+                        const uint64_t t2 =
+                            f2_add(f2_pack(__uint_as_float(dpv[e]), __uint_as_float(dpv[e + 1])), f2_pack(q.z, q.w));
+                        float d0, d1;
+                        f2_unpack(f2_mul(pp, t2), d0, d1);
+                        pk[e / 2] = cvt_bf16x2(p0, p1);
+                        dk2[e / 2] = cvt_bf16x2(d0, d1);
                     }
-                    const uint64_t pp = f2_pack(p0, p1);
-                    const uint64_t t2 =
-                        f2_add(f2_pack(__uint_as_float(dpv[e]), __uint_as_float(dpv[e + 1])), f2_pack(q.z, q.w));
-                    float d0, d1;
-                    f2_unpack(f2_mul(pp, t2), d0, d1);
-                    pk[e / 2] = cvt_bf16x2(p0, p1);
-                    dk2[e / 2] = cvt_bf16x2(d0, d1);
-                }
+                };
+                if (open) columns(std::false_type{});
+                else columns(std::true_type{});
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     const uint32_t off = sw128_offset(t, half * 4 + q4);
