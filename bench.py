@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "521ac9082c101078"): 821543936 + 479842048,
-    ("global_bwd", "521ac9082c101078"): 428666112 + 294057472,
+    ("local_bwd", "51d923c08c793564"): 821816832 + 479825920,
+    ("global_bwd", "51d923c08c793564"): 416202496 + 286070784,
 }
 
 
