@@ -419,6 +419,30 @@ def native_arm(a, rank, world, local_rank, dist_on):
                                         "ideal_speedup": dense_flops / max(fl_global, 1)}
         del dl
 
+    # ---- device-resident routing loop (Sec. 3.2): threshold select with the
+    # threshold on the device, then the Eq. 11 update, on this workload's gates
+    from paper_2608_29539_gb300 import logo as L
+    b_dev = torch.tensor([0.5], dtype=torch.float32, device=dev)
+    f_dev = torch.empty((1,), dtype=torch.float32, device=dev)
+    rl_bufs = (torch.empty_like(layer.z), torch.empty_like(layer.pos), torch.empty_like(layer.cu_q),
+               torch.empty_like(layer.row_of), torch.empty_like(layer.n_sel))
+
+    def routing_step():
+        L.logo_select_device_threshold(x["p"], b_dev, *rl_bufs, workspace=layer.ws)
+        L.logo_budget_update(rl_bufs[4], w.B, w.T, w.ratio, 2.0 ** -11, b_dev, f_out=f_dev)
+
+    for _ in range(3):
+        routing_step()
+    torch.cuda.synchronize()
+    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    r0.record()
+    for _ in range(50):
+        routing_step()
+    r1.record()
+    torch.cuda.synchronize()
+    line["device_routing_loop"] = {"us_per_step": r0.elapsed_time(r1) / 50 * 1e3, "launches_per_step": 4,
+                                   "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
+
     # ---- end to end through host buffers
     if not a.no_e2e:
         host = {k: x[k].cpu().pin_memory() for k in ("qL", "kL", "vL", "qG", "kG", "vG", "p", "dO")}

@@ -108,6 +108,40 @@ LOGO_API int logo_select(const float* gate_p, logo_dims dims, int mode, float b_
                 int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* workspace, size_t workspace_bytes,
                 void* stream);
 
+/* logo_select_device_threshold -- logo_select in LOGO_SELECT_THRESHOLD mode
+ *   with the Eq. 7 threshold read by the kernels from DEVICE memory (b_th:
+ *   one float32, caller-owned), so that logo_budget_update can move it
+ *   between steps without a host round trip (Sec. 3.2, Budget Control).
+ *   Same outputs, workspace (logo_select_workspace_size) and guarantees as
+ *   logo_select in threshold mode with that value; b_th must not be written
+ *   while the call runs on the stream (stream order suffices). */
+LOGO_API int logo_select_device_threshold(const float* gate_p, logo_dims dims, const float* b_th, uint8_t* z,
+                int32_t* pos, int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total, void* workspace,
+                size_t workspace_bytes, void* stream);
+
+/* logo_budget_update -- the budget controller of Sec. 3.2 on the device.
+ *   Eq. 3: F = N / (B*T) with N = *n_sel_total (the count logo_select wrote;
+ *   every token of the batch counts as valid); Eq. 11:
+ *     b_th <- b_th + gamma * sign(F - rho),  sign(0) = 0,
+ *   so F > rho raises the threshold (fewer tokens next step) and F < rho
+ *   lowers it.  F and the sign are evaluated in double; b_th (device, one
+ *   float32, updated in place) and gamma are float32 and the update is one
+ *   float32 addition, so the trajectory is exact and reproducible.
+ * In : n_sel_total [1] int32 (device); rho in [0, 1]; gamma >= 0 finite.
+ * Out: b_th [1] float32 (device, read and written); f_out [1] float32
+ *      (device, optional: F as float32; NULL to skip).
+ * One single-thread launch on `stream`. */
+LOGO_API int logo_budget_update(const int32_t* n_sel_total, logo_dims dims, float rho, float gamma, float* b_th,
+                float* f_out, void* stream);
+
+/* logo_pmask_initial_threshold -- P-mask start value (Sec. 3.2 Progressive
+ *   Masking, App. C.1): 0.5 - gamma * pmask_steps, computed in double and
+ *   returned as float32.  While every token is selected (F = 1 > rho) Eq. 11
+ *   raises b_th by gamma per step, so it reaches the gate centre 0.5 when the
+ *   P-mask phase of pmask_steps steps ends; until then b_th < 0 < p_t selects
+ *   every token.  Host function, no device work. */
+LOGO_API float logo_pmask_initial_threshold(float gamma, long long pmask_steps);
+
 /* logo_select_noalloc -- logo_select for callers that cannot allocate.
  *   No counterpart in the paper: this is a deployment variant of logo_select.
  *   Some callers hold only their own input and output buffers and have no way

@@ -11,6 +11,8 @@ numpy arrays.  Each function names the passage of the paper it follows:
 * ``select_threshold``  -- Eq. 7, z_t = 1[p_t > b_th] (float32 compare)
 * ``select_ratio``      -- per-sequence top-k reading of the target ratio rho
 * ``compact``           -- the selected set I (Sec. 3.2) packed ascending (App. B)
+* ``budget_update``     -- Eq. 3 realised ratio and the Eq. 11 threshold update
+* ``pmask_threshold``   -- the P-mask start value of Sec. 3.2 / App. C.1
 * ``attn_fwd/attn_bwd`` -- Eq. 1 over C^w_t (Eq. 6, local) or C^inf_t (Eq. 8,
                            global, selected rows only)
 * ``combine_fwd/bwd``   -- Eq. 9 ContextNorm + Eq. 10 fusion
@@ -61,6 +63,11 @@ def _load():
             lib.oracle_select_ratio.argtypes = [_f32p, _int, _int, _int, _u8p]
             lib.oracle_compact.argtypes = [_u8p, _int, _int, _i32p, _i32p, _i32p]
             lib.oracle_compact.restype = _i64
+            lib.oracle_budget_update.argtypes = [_i64, _i64, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                                 ctypes.POINTER(ctypes.c_double)]
+            lib.oracle_budget_update.restype = ctypes.c_float
+            lib.oracle_pmask_threshold.argtypes = [ctypes.c_double, _i64]
+            lib.oracle_pmask_threshold.restype = ctypes.c_double
             lib.oracle_attn_fwd.argtypes = [_f32p, _f32p, _f32p, _int, _int, _int, _int, _int,
                                             _i64, _i32p, _i32p, _int, _i32p, _int, ctypes.c_double,
                                             _f64p, _f64p]
@@ -123,6 +130,20 @@ def compact(z):
     row_of = np.zeros((B, T), dtype=np.int32)
     n = int(_load().oracle_compact(z, B, T, pos, cu_q, row_of))
     return pos[:n].copy(), cu_q, row_of, n
+
+
+def budget_update(n_sel: int, n_valid: int, rho: float, gamma: float, b_th: float):
+    """Eq. 3 + Eq. 11: returns (new b_th as float32, F).  See oracle_budget_update."""
+    F = ctypes.c_double(0.0)
+    b = _load().oracle_budget_update(int(n_sel), int(n_valid), ctypes.c_float(np.float32(rho)),
+                                     ctypes.c_float(np.float32(gamma)), ctypes.c_float(np.float32(b_th)),
+                                     ctypes.byref(F))
+    return np.float32(b), float(F.value)
+
+
+def pmask_threshold(gamma: float, steps: int) -> float:
+    """P-mask start b_th,0 = 0.5 - gamma * S (Sec. 3.2, App. C.1), in double."""
+    return float(_load().oracle_pmask_threshold(float(gamma), int(steps)))
 
 
 # ------------------------------------------------------------------ attention

@@ -37,6 +37,27 @@ void oracle_select_threshold(const float* p, int64_t n, float b_th, uint8_t* z)
     for (int64_t i = 0; i < n; ++i) z[i] = (p[i] > b_th) ? 1 : 0;
 }
 
+/* Eq. 3 and Eq. 11 (Sec. 3.2, Budget Control): the realised ratio is
+ * F = n_sel / n_valid, and the threshold moves by gamma * sign(F - rho).
+ * F and the sign are evaluated in double from the integer counts; b_th and
+ * gamma are float32 (the precision of the gate and of the Eq. 7 compare) and
+ * the update is one float32 addition.  Returns the new b_th; *F_out = F. */
+float oracle_budget_update(int64_t n_sel, int64_t n_valid, float rho, float gamma, float b_th, double* F_out)
+{
+    const double F = (double)n_sel / (double)n_valid;
+    const double d = F - (double)rho;
+    const float sgn = d > 0.0 ? 1.0f : (d < 0.0 ? -1.0f : 0.0f);
+    const float step = gamma * sgn; /* exact: sgn is -1, 0 or +1 */
+    if (F_out) *F_out = F;
+    return b_th + step;
+}
+
+/* P-mask start (Sec. 3.2 Progressive Masking, App. C.1): b_th starts at the
+ * gate centre 0.5 minus the total drift of S steps at rate gamma, so that
+ * while every token is selected (F = 1 > rho) it reaches 0.5 after S steps.
+ * Computed in double. */
+double oracle_pmask_threshold(double gamma, int64_t steps) { return 0.5 - gamma * (double)steps; }
+
 /* Ratio mode: in each sequence the k tokens with the largest gate p_t are
  * selected; equal gates are ordered by lower position first.  This is the
  * per-sequence quantile reading of the target ratio rho (k = floor(rho*T)),

@@ -133,7 +133,8 @@ __device__ __forceinline__ void decide(float pv, bool ratio_mode, float b_th, co
 }
 
 __global__ void __launch_bounds__(kThreads) count_kernel(const float* __restrict__ p, int T, int nchunk,
-                                                         int ratio_mode, float b_th,
+                                                         int ratio_mode, float b_th_host,
+                                                         const float* __restrict__ b_th_dev,
                                                          const SeqThresh* __restrict__ th,
                                                          ChunkCounts* __restrict__ counts)
 {
@@ -142,6 +143,7 @@ __global__ void __launch_bounds__(kThreads) count_kernel(const float* __restrict
     const int t0 = c * kChunk + threadIdx.x * kPerThread;
     const float* pb = p + static_cast<int64_t>(b) * T;
     SeqThresh tb = ratio_mode ? th[b] : SeqThresh{0u, 0};
+    const float b_th = b_th_dev ? *b_th_dev : b_th_host;  // Eq. 7 threshold (device-resident if given)
     int ngt = 0, neq = 0;
 #pragma unroll
     for (int i = 0; i < kPerThread; ++i) {
@@ -198,7 +200,8 @@ __global__ void __launch_bounds__(kThreads) scan_kernel(const ChunkCounts* __res
 }
 
 __global__ void __launch_bounds__(kThreads) write_kernel(const float* __restrict__ p, int T, int nchunk,
-                                                         int ratio_mode, float b_th,
+                                                         int ratio_mode, float b_th_host,
+                                                         const float* __restrict__ b_th_dev,
                                                          const SeqThresh* __restrict__ th,
                                                          const ChunkPlan* __restrict__ plan,
                                                          uint8_t* __restrict__ z, int32_t* __restrict__ pos,
@@ -209,6 +212,7 @@ __global__ void __launch_bounds__(kThreads) write_kernel(const float* __restrict
     const int t0 = c * kChunk + threadIdx.x * kPerThread;
     const int64_t off = static_cast<int64_t>(b) * T;
     SeqThresh tb = ratio_mode ? th[b] : SeqThresh{0u, 0};
+    const float b_th = b_th_dev ? *b_th_dev : b_th_host;
     ChunkPlan pl = plan[static_cast<int64_t>(b) * nchunk + c];
     bool gt[kPerThread], eq[kPerThread];
     int neq = 0;
@@ -303,10 +307,33 @@ extern "C" int logo_select(const float* gate_p, logo_dims dims, int mode, float 
     const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
     if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
     dim3 grid(nchunk, dims.B);
-    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.counts);
+    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, nullptr, ws.th, ws.counts);
     scan_kernel<<<1, kThreads, 0, st>>>(ws.counts, dims.B, nchunk, ratio_mode, ws.th, ws.plan, cu_q, n_sel_total);
-    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.plan, z, pos,
+    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, nullptr, ws.th, ws.plan, z, pos,
                                             row_of);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+// Threshold mode with b_th read from device memory by the kernels, so that a
+// device-side budget controller (logo_budget_update, Eq. 11) can move the
+// threshold between steps without a host round trip.
+extern "C" int logo_select_device_threshold(const float* gate_p, logo_dims dims, const float* b_th, uint8_t* z,
+                                            int32_t* pos, int32_t* cu_q, int32_t* row_of, int32_t* n_sel_total,
+                                            void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (dims.B < 1 || dims.T < 1) return LOGO_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(dims.B) * dims.T > (1ll << 30)) return LOGO_ERR_UNSUPPORTED;
+    if (!gate_p || !b_th || !z || !pos || !cu_q || !row_of || !n_sel_total) return LOGO_ERR_INVALID_ARG;
+    const size_t need = select_ws_layout(dims, nullptr, nullptr);
+    if (!workspace || workspace_bytes < need) return LOGO_ERR_WORKSPACE;
+    SelectWs ws;
+    select_ws_layout(dims, static_cast<char*>(workspace), &ws);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int nchunk = (dims.T + kChunk - 1) / kChunk;
+    dim3 grid(nchunk, dims.B);
+    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, 0, 0.0f, b_th, ws.th, ws.counts);
+    scan_kernel<<<1, kThreads, 0, st>>>(ws.counts, dims.B, nchunk, 0, ws.th, ws.plan, cu_q, n_sel_total);
+    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, 0, 0.0f, b_th, ws.th, ws.plan, z, pos, row_of);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
@@ -362,9 +389,9 @@ extern "C" int logo_select_noalloc(const float* gate_p, logo_dims dims, int mode
     const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
     if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
     dim3 grid(nchunk, dims.B);
-    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.counts);
+    count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, nullptr, ws.th, ws.counts);
     scan_kernel<<<1, kThreads, 0, st>>>(ws.counts, dims.B, nchunk, ratio_mode, ws.th, ws.plan, cu_q, n_sel_total);
-    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, ws.th, ws.plan, z, pos,
+    write_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, nullptr, ws.th, ws.plan, z, pos,
                                             row_of);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }

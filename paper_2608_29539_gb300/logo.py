@@ -58,6 +58,9 @@ _SIGS = {
     "logo_select_workspace_size": (_c_size, [Dims]),
     "logo_select": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
     "logo_select_noalloc": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "logo_select_device_threshold": (_c_int, [_vp, Dims, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
+    "logo_budget_update": (_c_int, [_vp, Dims, _c_float, _c_float, _vp, _vp, _vp]),
+    "logo_pmask_initial_threshold": (_c_float, [_c_float, ctypes.c_longlong]),
     "logo_local_attn_fwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp]),
     "logo_local_attn_bwd_workspace_size": (_c_size, [Dims]),
     "logo_local_attn_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp,
@@ -167,6 +170,45 @@ def logo_select(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None
     _call("logo_select", _p(gate_p), dims, int(mode), float(b_th), float(ratio), _p(z), _p(pos), _p(cu_q),
           _p(row_of), _p(n_sel_total), _p(ws), nbytes, _stream())
     return z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_select_device_threshold(gate_p, b_th, z=None, pos=None, cu_q=None, row_of=None, n_sel_total=None,
+                                 workspace=None):
+    """Eq. 7 routing with the threshold read on the device from b_th (a
+    one-element float32 CUDA tensor).  Returns (z, pos, cu_q, row_of, n_sel_total)."""
+    _need(gate_p, torch.float32, "gate_p")
+    _need(b_th, torch.float32, "b_th", (1,))
+    B, T = gate_p.shape
+    dev = gate_p.device
+    dims = Dims(B, T, 1, 1, 64)
+    z = z if z is not None else torch.empty((B, T), dtype=torch.uint8, device=dev)
+    pos = pos if pos is not None else torch.empty((B * T,), dtype=torch.int32, device=dev)
+    cu_q = cu_q if cu_q is not None else torch.empty((B + 1,), dtype=torch.int32, device=dev)
+    row_of = row_of if row_of is not None else torch.empty((B, T), dtype=torch.int32, device=dev)
+    n_sel_total = n_sel_total if n_sel_total is not None else torch.empty((1,), dtype=torch.int32, device=dev)
+    nbytes = workspace_bytes("select", dims)
+    ws = _workspace(nbytes, dev, workspace)
+    _call("logo_select_device_threshold", _p(gate_p), dims, _p(b_th), _p(z), _p(pos), _p(cu_q), _p(row_of),
+          _p(n_sel_total), _p(ws), nbytes, _stream())
+    return z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_budget_update(n_sel_total, B: int, T: int, rho: float, gamma: float, b_th, f_out=None):
+    """Eq. 3 + Eq. 11 on the device: b_th (one-element float32 CUDA tensor) is
+    moved by gamma * sign(N / (B*T) - rho) in place; f_out (optional, same
+    kind) receives F.  Returns b_th."""
+    _need(n_sel_total, torch.int32, "n_sel_total", (1,))
+    _need(b_th, torch.float32, "b_th", (1,))
+    if f_out is not None:
+        _need(f_out, torch.float32, "f_out", (1,))
+    _call("logo_budget_update", _p(n_sel_total), Dims(int(B), int(T), 1, 1, 64), float(rho), float(gamma),
+          _p(b_th), _p(f_out), _stream())
+    return b_th
+
+
+def logo_pmask_initial_threshold(gamma: float, pmask_steps: int) -> float:
+    """P-mask start value 0.5 - gamma * steps (Sec. 3.2, App. C.1); host only."""
+    return float(lib().logo_pmask_initial_threshold(float(gamma), int(pmask_steps)))
 
 
 def logo_select_noalloc(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None, pos=None, cu_q=None,

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from paper_2608_29539_gb300 import build
@@ -70,6 +71,33 @@ def test_host_side_argument_checks(lib):
     # combine: eps must be positive
     assert L.logo_combine(fake, fake, fake, fake, fake, null, null, ctypes.c_float(0.0), fake, null, null, d,
                           null) == logo.LOGO_ERR_INVALID_ARG
+
+
+def test_budget_controller_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    import oracle
+    L = logo.lib()
+    d = logo.Dims(2, 300, 1, 1, 64)
+    null = None
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected before use
+    f = ctypes.c_float
+    assert L.logo_budget_update(null, d, f(0.5), f(0.01), fake, null, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_budget_update(fake, d, f(0.5), f(0.01), null, null, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_budget_update(fake, d, f(1.5), f(0.01), fake, null, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_budget_update(fake, d, f(0.5), f(-0.01), fake, null, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_budget_update(fake, d, f(0.5), f(float("inf")), fake, null, null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_budget_update(fake, logo.Dims(0, 300, 1, 1, 64), f(0.5), f(0.01), fake, null,
+                                null) == logo.LOGO_ERR_INVALID_ARG
+    ws = L.logo_select_workspace_size(d)
+    assert L.logo_select_device_threshold(fake, d, null, fake, fake, fake, fake, fake, fake, ws,
+                                          null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_select_device_threshold(fake, d, fake, fake, fake, fake, fake, fake, fake, 16,
+                                          null) == logo.LOGO_ERR_WORKSPACE
+    # the P-mask start is a host function: against the oracle and App. C.1's value
+    for gamma, steps in ((0.0005, 5000), (2.0 ** -11, 4096), (0.01, 0), (0.003, 1234)):
+        got = logo.logo_pmask_initial_threshold(gamma, steps)
+        assert got == float(np.float32(oracle.pmask_threshold(float(np.float32(gamma)), steps)))
+    assert logo.logo_pmask_initial_threshold(0.0005, 5000) == -2.0
 
 
 def test_workspace_sizes_grow_with_shape(lib):

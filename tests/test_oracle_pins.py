@@ -48,6 +48,63 @@ def test_pmask_start_selects_everything():
     assert not oracle.select_threshold(p, 1.0).any()
 
 
+def test_pmask_start_value_of_app_c1():
+    g = json.load(open(os.path.join(GOLDEN, "pmask_threshold.json")))
+    assert oracle.pmask_threshold(g["gamma"], g["S"]) == pytest.approx(g["b_th0"], abs=1e-12)
+
+
+def test_budget_update_moves_the_threshold_as_sec32_states():
+    # Sec. 3.2: F > rho raises b_th (fewer tokens), F < rho lowers it; Eq. 3 F = N / |B|
+    g = 2.0 ** -11
+    b, F = oracle.budget_update(6, 10, 0.5, g, 0.25)
+    assert F == 0.6 and b > np.float32(0.25) and b - np.float32(0.25) == np.float32(g)
+    b, F = oracle.budget_update(4, 10, 0.5, g, 0.25)
+    assert F == 0.4 and b < np.float32(0.25) and np.float32(0.25) - b == np.float32(g)
+    b, F = oracle.budget_update(5, 10, 0.5, g, 0.25)  # F == rho exactly: sign(0) = 0
+    assert F == 0.5 and b == np.float32(0.25)
+    b, F = oracle.budget_update(0, 7, 0.0, g, 0.25)   # nothing selected at rho = 0: no move
+    assert F == 0.0 and b == np.float32(0.25)
+
+
+def test_pmask_phase_ends_at_the_gate_centre():
+    # Sec. 3.2 / App. C.1: from the P-mask start every token is selected while
+    # b_th < 0 < p (F = 1), and with the gates spread over (0, 1) F stays above
+    # rho = 0.25 all the way up, so each step raises b_th by gamma and it reaches
+    # the gate centre 0.5 after S steps.  gamma = 2^-11 and S = 4096 keep every
+    # value a multiple of 2^-11 below 2 in magnitude, so float32 is exact here.
+    gamma, S = 2.0 ** -11, 4096
+    b = np.float32(oracle.pmask_threshold(gamma, S))
+    assert b == np.float32(-1.5)
+    p = np.linspace(0.001, 0.999, 777, dtype=np.float32).reshape(1, -1)
+    for step in range(S):
+        z = oracle.select_threshold(p, b)
+        n = int(z.sum())
+        if b < 0:
+            assert n == p.size  # P-mask: every token takes the global branch
+        b, F = oracle.budget_update(n, p.size, 0.25, gamma, b)
+        assert F > 0.25
+    assert b == np.float32(0.5)
+
+
+def test_controller_settles_at_the_rho_quantile():
+    # Gates on a uniform grid p_t = (t + 0.5) / T: F(b) = #{p > b} / T = 1 - b up to
+    # 1/T, so Eq. 11 drives b_th to the (1 - rho) quantile and then stays within
+    # gamma (+ 1/T) of it, with F within the same distance of rho.  A sign error
+    # in the update runs away instead.
+    T, rho, gamma = 1000, 0.3, 2.0 ** -10
+    p = ((np.arange(T) + 0.5) / T).astype(np.float32).reshape(1, -1)
+    b = np.float32(0.5)
+    tail = []
+    for step in range(1200):
+        n = int(oracle.select_threshold(p, b).sum())
+        b, F = oracle.budget_update(n, T, rho, gamma, b)
+        if step >= 1000:
+            tail.append((float(b), F))
+    assert all(abs(bb - (1 - rho)) <= gamma + 1.0 / T for bb, _ in tail)
+    assert all(abs(F - rho) <= gamma + 2.0 / T for _, F in tail)
+    assert len({bb for bb, _ in tail}) >= 2  # it oscillates around the target
+
+
 def test_tiny_workload_selects_exactly_128():
     from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
     x = make_inputs(WORKLOADS["tiny"])
