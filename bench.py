@@ -61,6 +61,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     return ap.parse_args()
 
@@ -328,6 +329,68 @@ def config_of(w):
                 w.B * w.T * w.Hq * w.D * 2 / 2**20)}
 
 
+def decode_bench(dev, pk):
+    """Time one decoding step's attention (local branch from ring caches, global
+    branch for the selected sequences only, fusion) and the same step under the
+    paper's dense policy (every sequence runs the global call).  Inputs are
+    synthetic and seeded; the caches are larger than L2."""
+    from paper_2608_29539_gb300 import logo as L
+    B, Lc, Hq, Hkv, D, W = 32, 16384, 32, 8, 128, 1024
+    g = torch.Generator(device=dev).manual_seed(9)
+    kG = torch.randn((B, Lc, Hkv, D), generator=g, device=dev).to(torch.bfloat16)
+    vG = torch.randn((B, Lc, Hkv, D), generator=g, device=dev).to(torch.bfloat16)
+    kR = torch.randn((B, W, Hkv, D), generator=g, device=dev).to(torch.bfloat16)
+    vR = torch.randn((B, W, Hkv, D), generator=g, device=dev).to(torch.bfloat16)
+    qL = torch.randn((B, Hq, D), generator=g, device=dev).to(torch.bfloat16)
+    qG = torch.randn((B, Hq, D), generator=g, device=dev).to(torch.bfloat16)
+    seq_len = torch.full((B,), Lc, dtype=torch.int32, device=dev)
+    p = torch.rand((B, 1), generator=g, device=dev)
+    b_th = float(torch.quantile(p.flatten().cpu(), 7.0 / 8.0))
+    sparse_sel = L.logo_select(p, L.LOGO_SELECT_THRESHOLD, b_th=b_th)
+    dense_sel = L.logo_select(p, L.LOGO_SELECT_THRESHOLD, b_th=-1.0)
+    n = int(sparse_sel[4][0])
+    ws = torch.empty(int(L.lib().logo_decode_workspace_size(L.Dims(B, Lc, Hq, Hkv, D))), dtype=torch.uint8,
+                     device=dev)
+    o_l = torch.empty((B, Hq, D), dtype=torch.bfloat16, device=dev)
+    o_c = torch.empty((B, Hq, D), dtype=torch.bfloat16, device=dev)
+    o = torch.empty((B, 1, Hq, D), dtype=torch.bfloat16, device=dev)
+    rl = torch.empty((B, 1, Hq), dtype=torch.float32, device=dev)
+    rg = torch.empty((B, Hq), dtype=torch.float32, device=dev)
+
+    def step(sel):
+        zz, _, cq, ro, ns = sel
+        L.logo_decode_local_attn(qL, kR, vR, seq_len, W, o=o_l, workspace=ws)
+        L.logo_decode_global_sparse_attn(qG, kG, vG, seq_len, cq, ns, o_c=o_c, workspace=ws)
+        L.logo_combine(o_l.view(B, 1, Hq, D), o_c, p, zz, ro, None, None, 1e-6, o, rl, rg)
+
+    def timed(sel, reps=20):
+        for _ in range(3):
+            step(sel)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            step(sel)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    sparse_ms = timed(sparse_sel)
+    dense_ms = timed(dense_sel)
+    row_bytes = Hkv * D * 2 * 2  # K and V of one position, bf16
+    bytes_sparse = B * W * row_bytes + n * Lc * row_bytes
+    bytes_dense = B * W * row_bytes + B * Lc * row_bytes
+    gbs = bytes_sparse / (sparse_ms / 1e3) / 1e9
+    gbs_dense = bytes_dense / (dense_ms / 1e3) / 1e9
+    del kG, vG
+    return {"workload": f"B{B} cache {Lc} Hq{Hq}/Hkv{Hkv} d{D} W{W}, {n}/{B} sequences selected",
+            "ms_per_step": sparse_ms, "cache_GB_per_s": gbs, "frac_of_hbm_peak": gbs / pk["hbm"],
+            "dense_policy_ms": dense_ms, "dense_policy_GB_per_s": gbs_dense,
+            "speedup_vs_dense_policy": dense_ms / sparse_ms, "ideal_speedup": bytes_dense / bytes_sparse,
+            "launches_per_step": 6,
+            "note": "routing on (B, 1) is outside the timed loop; bytes = K and V cache rows read"}
+
+
 def native_arm(a, rank, world, local_rank, dist_on):
     from paper_2608_29539_gb300 import logo as L
     w = workload_named(a.workload)
@@ -442,6 +505,11 @@ def native_arm(a, rank, world, local_rank, dist_on):
     torch.cuda.synchronize()
     line["device_routing_loop"] = {"us_per_step": r0.elapsed_time(r1) / 50 * 1e3, "launches_per_step": 4,
                                    "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
+
+    # ---- one decoding step (Sec. 3.3): 32 sequences with 16K-token caches,
+    # GQA 32/8, d = 128, W = 1024, about 1/8 of the new tokens selected
+    if not a.no_decode and rank == 0:
+        line["decode"] = decode_bench(dev, pk)
 
     # ---- end to end through host buffers
     if not a.no_e2e:

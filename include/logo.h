@@ -142,6 +142,42 @@ LOGO_API int logo_budget_update(const int32_t* n_sel_total, logo_dims dims, floa
  *   every token.  Host function, no device work. */
 LOGO_API float logo_pmask_initial_threshold(float gamma, long long pmask_steps);
 
+/* logo_decode_workspace_size / logo_decode_local_attn /
+ * logo_decode_global_sparse_attn -- one autoregressive decoding step
+ *   (Sec. 3.3 Autoregressive Decoding): each of the B sequences has one new
+ *   token whose queries are q [B, Hq, D] (the local-branch queries for the
+ *   local call, the global-branch queries for the global call) and
+ *   seq_len[b] >= 1 tokens in its caches, the new one included, so the new
+ *   token sits at position seq_len[b] - 1.  The gate and routing of the step
+ *   come from logo_select (or logo_select_device_threshold) run on dims
+ *   (B, T = 1), and the two outputs are fused by logo_combine on dims
+ *   (B, T = 1): the same calls as in prefill.
+ *   local : Eq. 6 for the new token: the keys at positions
+ *           [max(0, len - W), len - 1], read from ring caches k_ring, v_ring
+ *           [B, R, Hkv, D] with R = dims.T >= W slots, position s in slot
+ *           s mod R.  Out: o [B, Hq, D].
+ *   global: Eq. 8 for the selected sequences only: packed row r (the r-th
+ *           selected sequence b, ascending; cu_q [B+1] and n_sel_total [1]
+ *           from the selection, device) attends positions [0, len - 1] of its
+ *           dense caches k_cache, v_cache [B, L, Hkv, D], L = dims.T >= len.
+ *           Out: o_c [B, Hq, D], packed rows; rows >= n_sel_total are left
+ *           untouched.  The work of unselected sequences is never launched
+ *           (the device-side count bounds it), so they read none of their
+ *           cache (the compaction the paper names as the missing serving
+ *           kernel) and no host synchronisation is needed.
+ *   Cache rows the step does not see (past seq_len, outside the window) may
+ *   hold anything.  dims: B, T = R or L, Hq, Hkv (Hq / Hkv <= 16), D in
+ *   {64, 128}; window >= 1 (local); scale as elsewhere (0 = 1/sqrt(D)).
+ *   Workspace: logo_decode_workspace_size(dims) bytes (per-chunk fp32
+ *   partials), one workspace per call in flight. */
+LOGO_API size_t logo_decode_workspace_size(logo_dims dims);
+LOGO_API int logo_decode_local_attn(const logo_bf16* q, const logo_bf16* k_ring, const logo_bf16* v_ring,
+                const int32_t* seq_len, logo_bf16* o, logo_dims dims, int window, float scale, void* workspace,
+                size_t workspace_bytes, void* stream);
+LOGO_API int logo_decode_global_sparse_attn(const logo_bf16* q, const logo_bf16* k_cache, const logo_bf16* v_cache,
+                const int32_t* seq_len, const int32_t* cu_q, const int32_t* n_sel_total, logo_bf16* o_c,
+                logo_dims dims, float scale, void* workspace, size_t workspace_bytes, void* stream);
+
 /* logo_select_noalloc -- logo_select for callers that cannot allocate.
  *   No counterpart in the paper: this is a deployment variant of logo_select.
  *   Some callers hold only their own input and output buffers and have no way

@@ -39,5 +39,6 @@ int select_tu_status(int clear);
 int combine_tu_status(int clear);
 int attn_fwd_tu_status(int clear);
 int attn_bwd_tu_status(int clear);
+int decode_tu_status(int clear);
 
 }  // namespace logo

@@ -61,6 +61,10 @@ _SIGS = {
     "logo_select_device_threshold": (_c_int, [_vp, Dims, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
     "logo_budget_update": (_c_int, [_vp, Dims, _c_float, _c_float, _vp, _vp, _vp]),
     "logo_pmask_initial_threshold": (_c_float, [_c_float, ctypes.c_longlong]),
+    "logo_decode_workspace_size": (_c_size, [Dims]),
+    "logo_decode_local_attn": (_c_int, [_vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp, _c_size, _vp]),
+    "logo_decode_global_sparse_attn": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_float, _vp, _c_size,
+                                                _vp]),
     "logo_local_attn_fwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp]),
     "logo_local_attn_bwd_workspace_size": (_c_size, [Dims]),
     "logo_local_attn_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _c_int, _c_float, _vp,
@@ -209,6 +213,48 @@ def logo_budget_update(n_sel_total, B: int, T: int, rho: float, gamma: float, b_
 def logo_pmask_initial_threshold(gamma: float, pmask_steps: int) -> float:
     """P-mask start value 0.5 - gamma * steps (Sec. 3.2, App. C.1); host only."""
     return float(lib().logo_pmask_initial_threshold(float(gamma), int(pmask_steps)))
+
+
+def _decode_dims(q, k):
+    B, Hq, D = q.shape
+    return Dims(B, k.shape[1], Hq, k.shape[2], D)
+
+
+def logo_decode_local_attn(q, k_ring, v_ring, seq_len, window: int, scale: float = 0.0, o=None, workspace=None):
+    """One decoding step of the local branch (Eq. 6) from ring caches
+    [B, R, Hkv, D] (position s in slot s mod R).  q [B, Hq, D]; seq_len [B]
+    int32 (cache length, the new token included).  Returns o [B, Hq, D]."""
+    _need(q, torch.bfloat16, "q")
+    _need(k_ring, torch.bfloat16, "k_ring")
+    _need(v_ring, torch.bfloat16, "v_ring", k_ring.shape)
+    _need(seq_len, torch.int32, "seq_len", (q.shape[0],))
+    dims = _decode_dims(q, k_ring)
+    o = o if o is not None else torch.empty_like(q)
+    nbytes = int(lib().logo_decode_workspace_size(dims))
+    ws = _workspace(nbytes, q.device, workspace)
+    _call("logo_decode_local_attn", _p(q), _p(k_ring), _p(v_ring), _p(seq_len), _p(o), dims, int(window),
+          float(scale), _p(ws), nbytes, _stream())
+    return o
+
+
+def logo_decode_global_sparse_attn(q, k_cache, v_cache, seq_len, cu_q, n_sel_total, scale: float = 0.0, o_c=None,
+                                   workspace=None):
+    """One decoding step of the global branch (Eq. 8) for the selected
+    sequences only (packed rows of a (B, 1) selection), from dense caches
+    [B, L, Hkv, D].  Returns o_c [B, Hq, D] (packed rows; rows >= n_sel untouched)."""
+    _need(q, torch.bfloat16, "q")
+    _need(k_cache, torch.bfloat16, "k_cache")
+    _need(v_cache, torch.bfloat16, "v_cache", k_cache.shape)
+    _need(seq_len, torch.int32, "seq_len", (q.shape[0],))
+    _need(cu_q, torch.int32, "cu_q", (q.shape[0] + 1,))
+    _need(n_sel_total, torch.int32, "n_sel_total", (1,))
+    dims = _decode_dims(q, k_cache)
+    o_c = o_c if o_c is not None else torch.empty_like(q)
+    nbytes = int(lib().logo_decode_workspace_size(dims))
+    ws = _workspace(nbytes, q.device, workspace)
+    _call("logo_decode_global_sparse_attn", _p(q), _p(k_cache), _p(v_cache), _p(seq_len), _p(cu_q),
+          _p(n_sel_total), _p(o_c), dims, float(scale), _p(ws), nbytes, _stream())
+    return o_c
 
 
 def logo_select_noalloc(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None, pos=None, cu_q=None,

@@ -100,6 +100,31 @@ def test_budget_controller_host_checks(lib):
     assert logo.logo_pmask_initial_threshold(0.0005, 5000) == -2.0
 
 
+def test_decode_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    d = logo.Dims(4, 2048, 8, 2, 128)
+    null = None
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected before use
+    f = ctypes.c_float
+    ws = L.logo_decode_workspace_size(d)
+    assert ws >= 4 * 8 * 16 * 130 * 4
+    assert L.logo_decode_workspace_size(logo.Dims(4, 2048, 64, 2, 128)) == 0  # group of 32 > 16
+    assert L.logo_decode_local_attn(null, fake, fake, fake, fake, d, 1024, f(0.0), fake, ws,
+                                    null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_decode_local_attn(fake, fake, fake, fake, fake, d, 0, f(0.0), fake, ws,
+                                    null) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_decode_local_attn(fake, fake, fake, fake, fake, d, 1024, f(0.0), fake, 16,
+                                    null) == logo.LOGO_ERR_WORKSPACE
+    assert L.logo_decode_local_attn(fake, fake, fake, fake, fake, logo.Dims(4, 2048, 8, 2, 96), 1024, f(0.0), fake,
+                                    ws, null) == logo.LOGO_ERR_UNSUPPORTED
+    assert L.logo_decode_global_sparse_attn(fake, fake, fake, fake, null, fake, fake, d, f(0.0), fake, ws,
+                                            null) == logo.LOGO_ERR_INVALID_ARG
+    odd = ctypes.c_void_p((1 << 20) + 2)
+    assert L.logo_decode_global_sparse_attn(odd, fake, fake, fake, fake, fake, fake, d, f(0.0), fake, ws,
+                                            null) == logo.LOGO_ERR_UNSUPPORTED
+
+
 def test_workspace_sizes_grow_with_shape(lib):
     from paper_2608_29539_gb300 import logo
     L = logo.lib()
