@@ -67,6 +67,7 @@ struct BwdParams {
     const int32_t* pos;
     const int32_t* cu_q;
     const int32_t* first_row;  // global: [B, nblk] first packed row of sequence b whose position reaches block j
+    logo_bf16* dq_fill;        // global, d = 128: dense dQ [B, T, Hq, D] whose unselected rows this kernel zeroes
     int B, T, Hq, Hkv, window, cap, nblk, q_tiles;
     float scale, scale_log2;
 };
@@ -458,7 +459,7 @@ struct Bwd2Cfg {
     static constexpr uint32_t kColDV = 128;
     static constexpr uint32_t kColBuf = 256;  // buffer b: S^T at 256+128b (64 cols), dP^T at +64
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr int kThreads = 448;
+    static constexpr int kThreads = 480;
 };
 
 template <bool GLOBAL>
@@ -779,7 +780,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 mbar_arrive(smem_u32(&bar_ds_full[b]));
             }
         }
-    } else {
+    } else if (warp < 14) {
         // ------------------------------------------------------------ dQ drain, dK/dV epilogue
         const int quad = warp & 3;
         const int t = quad * 32 + lane;  // head-dim row of dQ^T; key row of dK/dV
@@ -857,6 +858,38 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             tc_fence_before();
             mbar_arrive(smem_u32(&bar_dkv_empty));
             ++kv_items;
+        }
+    } else if (GLOBAL && p.dq_fill) {
+        // ------------------------------------------------------------ dQ zero fill
+        // warp 14: zero the dense dQ rows of the tokens that were not selected
+        // (the conversion after this kernel writes only the selected rows).  This
+        // kernel leaves nearly all of HBM's bandwidth idle; a separate pass
+        // writing the whole dense tensor would not.
+        const int64_t ntok = static_cast<int64_t>(p.B) * p.T;
+        const int64_t per = (ntok + gridDim.x - 1) / gridDim.x;
+        const int64_t t_begin = static_cast<int64_t>(blockIdx.x) * per;
+        const int64_t t_end = t_begin + per < ntok ? t_begin + per : ntok;
+        const int row_vecs = p.Hq * D / 8;  // 16-byte vectors per token row
+        int cur_b = -1, r = 0, r_hi = 0;
+        for (int64_t bt = t_begin; bt < t_end; ++bt) {
+            const int b = static_cast<int>(bt / p.T), t = static_cast<int>(bt % p.T);
+            if (b != cur_b) {  // first packed row of sequence b at or after position t
+                cur_b = b;
+                int lo = p.cu_q[b], hi = p.cu_q[b + 1];
+                r_hi = hi;
+                while (lo < hi) {
+                    const int mid = (lo + hi) >> 1;
+                    if (p.pos[mid] < t) lo = mid + 1;
+                    else hi = mid;
+                }
+                r = lo;
+            }
+            if (r < r_hi && p.pos[r] == t) {  // selected: converted later
+                ++r;
+                continue;
+            }
+            uint4* dst = reinterpret_cast<uint4*>(p.dq_fill + bt * p.Hq * D);
+            for (int v = lane; v < row_vecs; v += 32) dst[v] = make_uint4(0u, 0u, 0u, 0u);
         }
     }
     tc_fence_before();
@@ -937,6 +970,32 @@ __global__ void __launch_bounds__(256) first_row_kernel(const int32_t* __restric
         else hi = mid;
     }
     first_row[idx] = lo;
+}
+
+// Global branch, d = 128: dQ accumulator rows of the selected tokens -> their
+// rows of the dense dq (the backward kernel zeroed the others).  One block per
+// packed row; blocks past the selected count return.
+__global__ void __launch_bounds__(128) bwd_post_selected_kernel(const float* __restrict__ dq_acc,
+                                                                const int32_t* __restrict__ pos,
+                                                                const int32_t* __restrict__ cu_q,
+                                                                const int32_t* __restrict__ n_sel, int B, int T, int H,
+                                                                int D, logo_bf16* __restrict__ dq)
+{
+    const int r = blockIdx.x;
+    if (r >= *n_sel) return;
+    const int b = seq_of_row(cu_q, B, r);
+    const int64_t dst_row = static_cast<int64_t>(b) * T + pos[r];
+    const int row_elems = H * D;
+    for (int v = threadIdx.x; v < row_elems / 8; v += blockDim.x) {
+        const float4* s = reinterpret_cast<const float4*>(dq_acc + static_cast<int64_t>(r) * row_elems + v * 8);
+        const float4 a = s[0], c = s[1];
+        uint4 w;
+        w.x = pack_bf16x2(a.x, a.y);
+        w.y = pack_bf16x2(a.z, a.w);
+        w.z = pack_bf16x2(c.x, c.y);
+        w.w = pack_bf16x2(c.z, c.w);
+        *reinterpret_cast<uint4*>(dq + dst_row * row_elems + v * 8) = w;
+    }
 }
 
 // dQ accumulator (fp32) -> dq (bf16).  Local: elementwise.  Global: every
@@ -1166,6 +1225,7 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     prm.pos = pos;
     prm.cu_q = cu_q;
     prm.first_row = ws.first_row;
+    prm.dq_fill = dims.D == 128 ? dq : nullptr;
     prm.B = dims.B;
     prm.T = dims.T;
     prm.Hq = dims.Hq;
@@ -1178,6 +1238,10 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     prm.scale_log2 = scale * kLog2e;
     rc = dims.D == 128 ? launch_bwd<128, true>(prm, st) : launch_bwd<64, true>(prm, st);
     if (rc != LOGO_OK) return rc;
-    bwd_post_kernel<true><<<cap, 128, 0, st>>>(ws.dq_acc, pos, cu_q, dims.T, dims.Hq, dims.D, dq);
+    if (dims.D == 128)
+        bwd_post_selected_kernel<<<cap, 128, 0, st>>>(ws.dq_acc, pos, cu_q, n_sel_total, dims.B, dims.T, dims.Hq,
+                                                      dims.D, dq);
+    else
+        bwd_post_kernel<true><<<cap, 128, 0, st>>>(ws.dq_acc, pos, cu_q, dims.T, dims.Hq, dims.D, dq);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }

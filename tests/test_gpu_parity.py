@@ -197,7 +197,9 @@ def test_global_bwd(B, T, Hq, Hkv, D, kind, ratio):
     dO_c[:n] = seeded((n, Hq, D), 77 + T, torch.bfloat16)
     qc, kc, vc = q.cuda(), k.cuda(), v.cuda()
     o_c, lse_c = L().logo_global_sparse_attn_fwd(qc, kc, vc, pos, cu_q, nt)
-    dq, dk, dv = L().logo_global_sparse_attn_bwd(qc, kc, vc, pos, cu_q, nt, o_c, lse_c, dO_c.cuda())
+    # dq starts poisoned: every row, selected or not, must be written by the call
+    dq0 = torch.full(qc.shape, float("nan"), dtype=torch.bfloat16, device=qc.device)
+    dq, dk, dv = L().logo_global_sparse_attn_bwd(qc, kc, vc, pos, cu_q, nt, o_c, lse_c, dO_c.cuda(), dq=dq0)
     torch.cuda.synchronize()
     rb, rt = oracle.global_rows(opos, ocu)
     rdq_c, rdk, rdv = oracle.attn_bwd(np32(q), np32(k), np32(v), rb, rt, 0, np32(dO_c[:n]))
