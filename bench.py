@@ -157,7 +157,7 @@ def make_device_inputs(w, device):
 
 CALLS = ["select", "local_fwd", "global_fwd", "combine", "combine_bwd", "global_bwd", "local_bwd"]
 LAUNCHES_PER_STEP = {"select": 4, "local_fwd": 1, "global_fwd": 3, "combine": 1, "combine_bwd": 1,
-                     "global_bwd": 5, "local_bwd": 3}
+                     "global_bwd": 3, "local_bwd": 3}
 
 
 def run_step(layer, g, ev=None):

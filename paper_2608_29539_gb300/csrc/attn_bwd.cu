@@ -902,20 +902,57 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
 
 // ---------------------------------------------------------------- pre / post
 // Per (row, head): Dsum = sum_d dO * O (fp32); zero the dQ accumulator rows.
-// Global branch: also copy dO_c into the workspace, zero-padding the 128 rows
-// after the last selected one so that partial tiles read finite values.
+// Global branch: also copy dO_c into the workspace and gather the selected
+// rows of the dense Q into the packed layout (App. B), zero-padding the 128
+// rows after the last selected one so that partial tiles read finite values;
+// and build, for every sequence b and KV block j, the first packed row of b
+// whose position reaches the block's first key (App. B's precomputed search
+// that lets the backward skip every query tile before it).
+struct GlobalPrep {
+    const logo_bf16* q;   // dense [B, T, H, D]
+    const int32_t* pos;
+    const int32_t* cu_q;
+    logo_bf16* qc;        // packed [cap + 128, H, D]
+    int32_t* first_row;   // [B, nblk]
+    int B, nblk;
+};
+
 template <bool GLOBAL>
 __global__ void __launch_bounds__(128) bwd_pre_kernel(const logo_bf16* __restrict__ o, const logo_bf16* __restrict__ dO,
                                                       const int32_t* __restrict__ n_sel, int rows_host, int T, int H,
                                                       int D, int cap, float* __restrict__ dsum,
-                                                      logo_bf16* __restrict__ do_copy, float* __restrict__ dq_acc)
+                                                      logo_bf16* __restrict__ do_copy, float* __restrict__ dq_acc,
+                                                      GlobalPrep gp)
 {
     const int n = GLOBAL ? *n_sel : rows_host;
     const int rows = GLOBAL ? n + kBM : rows_host;
     const int vpr = D / 8, nvec = H * vpr;
+    if (GLOBAL) {
+        for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < gp.B * gp.nblk; idx += gridDim.x * blockDim.x) {
+            const int b = idx / gp.nblk, j = idx % gp.nblk;
+            int lo = gp.cu_q[b], hi = gp.cu_q[b + 1];
+            const int k0 = j * kBN;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (gp.pos[mid] < k0) lo = mid + 1;
+                else hi = mid;
+            }
+            gp.first_row[idx] = lo;
+        }
+    }
     for (int row = blockIdx.x; row < rows; row += gridDim.x) {
         const bool live = row < n;
         const int64_t base = static_cast<int64_t>(row) * H * D;
+        if (GLOBAL) {
+            uint4* dst = reinterpret_cast<uint4*>(gp.qc + base);
+            if (live) {
+                const int b = seq_of_row(gp.cu_q, gp.B, row);
+                const uint4* src = reinterpret_cast<const uint4*>(gp.q + (static_cast<int64_t>(b) * T + gp.pos[row]) * H * D);
+                for (int v = threadIdx.x; v < nvec; v += blockDim.x) dst[v] = src[v];
+            } else {
+                for (int v = threadIdx.x; v < nvec; v += blockDim.x) dst[v] = make_uint4(0, 0, 0, 0);
+            }
+        }
         for (int v0 = 0; v0 < nvec; v0 += blockDim.x) {
             const int v = v0 + threadIdx.x;
             const bool active = v < nvec;
@@ -952,49 +989,30 @@ __global__ void __launch_bounds__(128) bwd_pre_kernel(const logo_bf16* __restric
     }
 }
 
-// For every sequence b and KV block j: the first packed row of b whose
-// position reaches the block's first key (App. B's precomputed search that
-// lets the backward skip every query tile before it).
-__global__ void __launch_bounds__(256) first_row_kernel(const int32_t* __restrict__ pos,
-                                                        const int32_t* __restrict__ cu_q, int B, int nblk,
-                                                        int32_t* __restrict__ first_row)
-{
-    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= B * nblk) return;
-    const int b = idx / nblk, j = idx % nblk;
-    int lo = cu_q[b], hi = cu_q[b + 1];
-    const int k0 = j * kBN;
-    while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (pos[mid] < k0) lo = mid + 1;
-        else hi = mid;
-    }
-    first_row[idx] = lo;
-}
-
 // Global branch, d = 128: dQ accumulator rows of the selected tokens -> their
-// rows of the dense dq (the backward kernel zeroed the others).  One block per
-// packed row; blocks past the selected count return.
+// rows of the dense dq (the backward kernel zeroed the others); blocks stride
+// over the packed rows below the selected count.
 __global__ void __launch_bounds__(128) bwd_post_selected_kernel(const float* __restrict__ dq_acc,
                                                                 const int32_t* __restrict__ pos,
                                                                 const int32_t* __restrict__ cu_q,
                                                                 const int32_t* __restrict__ n_sel, int B, int T, int H,
                                                                 int D, logo_bf16* __restrict__ dq)
 {
-    const int r = blockIdx.x;
-    if (r >= *n_sel) return;
-    const int b = seq_of_row(cu_q, B, r);
-    const int64_t dst_row = static_cast<int64_t>(b) * T + pos[r];
+    const int n = *n_sel;
     const int row_elems = H * D;
-    for (int v = threadIdx.x; v < row_elems / 8; v += blockDim.x) {
-        const float4* s = reinterpret_cast<const float4*>(dq_acc + static_cast<int64_t>(r) * row_elems + v * 8);
-        const float4 a = s[0], c = s[1];
-        uint4 w;
-        w.x = pack_bf16x2(a.x, a.y);
-        w.y = pack_bf16x2(a.z, a.w);
-        w.z = pack_bf16x2(c.x, c.y);
-        w.w = pack_bf16x2(c.z, c.w);
-        *reinterpret_cast<uint4*>(dq + dst_row * row_elems + v * 8) = w;
+    for (int r = blockIdx.x; r < n; r += gridDim.x) {
+        const int b = seq_of_row(cu_q, B, r);
+        const int64_t dst_row = static_cast<int64_t>(b) * T + pos[r];
+        for (int v = threadIdx.x; v < row_elems / 8; v += blockDim.x) {
+            const float4* s = reinterpret_cast<const float4*>(dq_acc + static_cast<int64_t>(r) * row_elems + v * 8);
+            const float4 a = s[0], c = s[1];
+            uint4 w;
+            w.x = pack_bf16x2(a.x, a.y);
+            w.y = pack_bf16x2(a.z, a.w);
+            w.z = pack_bf16x2(c.x, c.y);
+            w.w = pack_bf16x2(c.z, c.w);
+            *reinterpret_cast<uint4*>(dq + dst_row * row_elems + v * 8) = w;
+        }
     }
 }
 
@@ -1148,7 +1166,7 @@ extern "C" int logo_local_attn_bwd(const logo_bf16* q, const logo_bf16* k, const
     const int rows = dims.B * dims.T;
     const int pre_grid = max(1, min(rows, device_sm_count() * 16));
     bwd_pre_kernel<false><<<pre_grid, 128, 0, st>>>(o, dO, nullptr, rows, dims.T, dims.Hq, dims.D, 0, ws.dsum,
-                                                    nullptr, ws.dq_acc);
+                                                    nullptr, ws.dq_acc, GlobalPrep{});
     BwdParams prm{};
     const uint32_t qrows = dims.D == 128 ? Bwd2Cfg::kBQ : kBM;
     if (!encode_bf16_4d(&prm.tm_q, q, dims.D, dims.Hq, dims.T, dims.B, 64, qrows) ||
@@ -1202,13 +1220,11 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     global_bwd_ws_layout(dims, static_cast<char*>(workspace), &ws);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int cap = dims.B * dims.T;
-    const int row_elems = dims.Hq * dims.D;
     const int grid_rows = max(1, min(cap + kBM, device_sm_count() * 16));
-    gather_rows_kernel<<<grid_rows, 256, 0, st>>>(q, pos, cu_q, n_sel_total, dims.B, dims.T, row_elems, ws.qc);
-    bwd_pre_kernel<true><<<grid_rows, 128, 0, st>>>(o_c, dO_c, n_sel_total, 0, dims.T, dims.Hq, dims.D, cap, ws.dsum,
-                                                    ws.doc, ws.dq_acc);
     const int nblk = (dims.T + kBN - 1) / kBN;
-    first_row_kernel<<<(dims.B * nblk + 255) / 256, 256, 0, st>>>(pos, cu_q, dims.B, nblk, ws.first_row);
+    const GlobalPrep gp{q, pos, cu_q, ws.qc, ws.first_row, dims.B, nblk};
+    bwd_pre_kernel<true><<<grid_rows, 128, 0, st>>>(o_c, dO_c, n_sel_total, 0, dims.T, dims.Hq, dims.D, cap, ws.dsum,
+                                                    ws.doc, ws.dq_acc, gp);
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     BwdParams prm{};
     const uint32_t qrows = dims.D == 128 ? Bwd2Cfg::kBQ : kBM;
@@ -1239,8 +1255,8 @@ extern "C" int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* 
     rc = dims.D == 128 ? launch_bwd<128, true>(prm, st) : launch_bwd<64, true>(prm, st);
     if (rc != LOGO_OK) return rc;
     if (dims.D == 128)
-        bwd_post_selected_kernel<<<cap, 128, 0, st>>>(ws.dq_acc, pos, cu_q, n_sel_total, dims.B, dims.T, dims.Hq,
-                                                      dims.D, dq);
+        bwd_post_selected_kernel<<<grid_rows, 128, 0, st>>>(ws.dq_acc, pos, cu_q, n_sel_total, dims.B, dims.T,
+                                                            dims.Hq, dims.D, dq);
     else
         bwd_post_kernel<true><<<cap, 128, 0, st>>>(ws.dq_acc, pos, cu_q, dims.T, dims.Hq, dims.D, dq);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
