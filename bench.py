@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "51d923c08c793564"): 821816832 + 479825920,
-    ("global_bwd", "51d923c08c793564"): 416202496 + 286070784,
+    ("local_bwd", "84c8e7a80b76632d"): 821894400 + 479746304,
+    ("global_bwd", "84c8e7a80b76632d"): 464744960 + 429653248,
 }
 
 
@@ -62,6 +62,7 @@ def parse():
     ap.add_argument("--no-dense", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-routing", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     return ap.parse_args()
 
@@ -329,6 +330,32 @@ def config_of(w):
                 w.B * w.T * w.Hq * w.D * 2 / 2**20)}
 
 
+def routing_bench(layer, x, w, dev):
+    """Device-resident routing loop: logo_select_device_threshold then
+    logo_budget_update, 50 steps on the workload's gates, no host sync."""
+    from paper_2608_29539_gb300 import logo as L
+    b_dev = torch.tensor([0.5], dtype=torch.float32, device=dev)
+    f_dev = torch.empty((1,), dtype=torch.float32, device=dev)
+    rl_bufs = (torch.empty_like(layer.z), torch.empty_like(layer.pos), torch.empty_like(layer.cu_q),
+               torch.empty_like(layer.row_of), torch.empty_like(layer.n_sel))
+
+    def routing_step():
+        L.logo_select_device_threshold(x["p"], b_dev, *rl_bufs, workspace=layer.ws)
+        L.logo_budget_update(rl_bufs[4], w.B, w.T, w.ratio, 2.0 ** -11, b_dev, f_out=f_dev)
+
+    for _ in range(3):
+        routing_step()
+    torch.cuda.synchronize()
+    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    r0.record()
+    for _ in range(50):
+        routing_step()
+    r1.record()
+    torch.cuda.synchronize()
+    return {"us_per_step": r0.elapsed_time(r1) / 50 * 1e3, "launches_per_step": 4,
+            "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
+
+
 def decode_bench(dev, pk):
     """Time one decoding step's attention (local branch from ring caches, global
     branch for the selected sequences only, fusion) and the same step under the
@@ -484,27 +511,8 @@ def native_arm(a, rank, world, local_rank, dist_on):
 
     # ---- device-resident routing loop (Sec. 3.2): threshold select with the
     # threshold on the device, then the Eq. 11 update, on this workload's gates
-    from paper_2608_29539_gb300 import logo as L
-    b_dev = torch.tensor([0.5], dtype=torch.float32, device=dev)
-    f_dev = torch.empty((1,), dtype=torch.float32, device=dev)
-    rl_bufs = (torch.empty_like(layer.z), torch.empty_like(layer.pos), torch.empty_like(layer.cu_q),
-               torch.empty_like(layer.row_of), torch.empty_like(layer.n_sel))
-
-    def routing_step():
-        L.logo_select_device_threshold(x["p"], b_dev, *rl_bufs, workspace=layer.ws)
-        L.logo_budget_update(rl_bufs[4], w.B, w.T, w.ratio, 2.0 ** -11, b_dev, f_out=f_dev)
-
-    for _ in range(3):
-        routing_step()
-    torch.cuda.synchronize()
-    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    r0.record()
-    for _ in range(50):
-        routing_step()
-    r1.record()
-    torch.cuda.synchronize()
-    line["device_routing_loop"] = {"us_per_step": r0.elapsed_time(r1) / 50 * 1e3, "launches_per_step": 4,
-                                   "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
+    if not a.no_routing:
+        line["device_routing_loop"] = routing_bench(layer, x, w, dev)
 
     # ---- one decoding step (Sec. 3.3): 32 sequences with 16K-token caches,
     # GQA 32/8, d = 128, W = 1024, about 1/8 of the new tokens selected
