@@ -3,13 +3,16 @@
 //   logo_local_attn_fwd          O^L = SoftmaxAttn_W(Q^L, K^L, V^L)   (Eq. 6)
 //   logo_global_sparse_attn_fwd  O^G_I = SoftmaxAttn_inf(Q^G_I, K^G, V^G) (Eq. 8)
 //
-// One persistent kernel template serves both.  A CTA (6 warps) loops over
+// One persistent kernel template serves both.  A CTA (7 warps) loops over
 // work items = (128-row query tile, query head):
 //   warp 0      TMA producer: Q tile once per item, then K/V blocks through a
 //               ring of shared-memory stages (128-byte swizzle).
-//   warp 1      MMA issuer (one thread): S = Q K^T into one of two TMEM S
-//               buffers, then O += P V into the TMEM O accumulator with P
-//               read straight from TMEM.
+//   warp 1      S issuer (one thread): S = Q K^T into one of two TMEM S buffers.
+//   warp 6      P.V issuer (one thread): O += P V into the TMEM O accumulator
+//               with P read straight from TMEM.  Two issuing threads keep the
+//               tensor pipe fed while either waits for its inputs: the issue
+//               queue is short, so a single thread that stops to wait starves
+//               the pipe (measured: 1728 vs 2427 TFLOP/s on the same MMA stream).
 //   warps 2..5  softmax: one thread per query row (its TMEM lane).  Online
 //               softmax in the log2 domain with conditional rescaling of O
 //               (only when the running max grows by more than 2^8); P goes
@@ -95,12 +98,12 @@ __device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
 }
 
 template <int D, bool GLOBAL>
-__global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
+__global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
 {
     using C = FwdCfg<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_drain;
+    __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_drain, bar_drain_pv;
     __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_v_full[C::kStages], bar_kv_empty[C::kStages];
     __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2], bar_p_full[2], bar_p_free[2];
     __shared__ uint32_t tmem_base_sh;
@@ -121,6 +124,7 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
         mbar_init(smem_u32(&bar_q_full), 1);
         mbar_init(smem_u32(&bar_q_empty), 1);
         mbar_init(smem_u32(&bar_drain), 1);
+        mbar_init(smem_u32(&bar_drain_pv), 1);
         for (int s = 0; s < C::kStages; ++s) {
             mbar_init(smem_u32(&bar_k_full[s]), 1);
             mbar_init(smem_u32(&bar_v_full[s]), 1);
@@ -128,7 +132,7 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
         }
         for (int s = 0; s < 4; ++s) {
             mbar_init(smem_u32(&bar_item_full[s]), 1);
-            mbar_init(smem_u32(&bar_item_empty[s]), 5);  // the MMA thread + one lane per softmax warp
+            mbar_init(smem_u32(&bar_item_empty[s]), 6);  // the two MMA threads + one lane per softmax warp
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_s_full[s]), 1);
@@ -228,30 +232,15 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+        // ------------------------------------------------------------ S issuer
+        // S = Q K^T of every block; the P.V products come from warp 6, so that
+        // neither stream's waits leave the tensor pipe without queued work
+        // (the issue queue is short: an issuing thread runs only a few
+        // instructions ahead of execution)
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBM, kBN, false, false);
-            constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, false, true);
             int kv_it = 0, s_it = 0, item_i = 0;
             bool ok = true;
-            auto issue_pv = [&](int jj) -> bool {
-                const int itg = s_it + jj;
-                const int st = (kv_it + jj) % C::kStages, f = (kv_it + jj) / C::kStages;
-                // per-buffer: the next arrival on this buffer needs this P.V done
-                if (!mbar_wait(smem_u32(&bar_p_full[itg & 1]), (itg >> 1) & 1, &abort_flag)) return false;
-                if (!mbar_wait(smem_u32(&bar_v_full[st]), f & 1, &abort_flag)) return false;
-                tc_fence_after();
-                const uint32_t vbase = sV + st * C::kTileBytes;
-                const uint32_t pcol = tmem + ((itg & 1) ? C::kColP1 : C::kColP0);
-#pragma unroll
-                for (int ks = 0; ks < kBN / 16; ++ks) {
-                    const uint64_t b = sdesc_sw128(vbase + ks * 2048, 16384, 1024);
-                    umma_bf16_ts(tmem + C::kColO, pcol + ks * 8, b, idPV, (jj > 0 || ks > 0) ? 1u : 0u);
-                }
-                umma_commit(smem_u32(&bar_p_free[itg & 1]));
-                umma_commit(smem_u32(&bar_kv_empty[st]));
-                return true;
-            };
             for (;; ++item_i) {
                 const int k = consume_item(item_i, &ok, false);
                 if (k < 0) break;
@@ -274,11 +263,9 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                                      ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_s_full[buf]));
-                    if (j > 0) ok = issue_pv(j - 1);
                 }
                 if (!ok) break;
                 umma_commit(smem_u32(&bar_q_empty));
-                if (!(ok = issue_pv(nblk - 1))) break;
                 kv_it += nblk;
                 s_it += nblk;
             }
@@ -287,7 +274,45 @@ __global__ void __launch_bounds__(192, 1) attn_fwd_kernel(const __grid_constant_
                 mbar_wait_drain(smem_u32(&bar_drain), 0);
             }
         }
-    } else {
+    } else if (warp == 6) {
+        // ------------------------------------------------------------ P.V issuer
+        if (lane == 0) {
+            constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, false, true);
+            int kv_it = 0, s_it = 0, item_i = 0;
+            bool ok = true;
+            for (;; ++item_i) {
+                const int k = consume_item(item_i, &ok, false);
+                if (k < 0) break;
+                const FwdItem it = decode_item<GLOBAL>(p, k);
+                const int nblk = it.blk_hi - it.blk_lo + 1;
+                for (int j = 0; j < nblk && ok; ++j) {
+                    const int itg = s_it + j;
+                    const int st = (kv_it + j) % C::kStages, f = (kv_it + j) / C::kStages;
+                    // P of this block written (which also orders this P.V after the
+                    // previous item's epilogue: the softmax warps wrote P later)
+                    if (!(ok = mbar_wait(smem_u32(&bar_p_full[itg & 1]), (itg >> 1) & 1, &abort_flag))) break;
+                    if (!(ok = mbar_wait(smem_u32(&bar_v_full[st]), f & 1, &abort_flag))) break;
+                    tc_fence_after();
+                    const uint32_t vbase = sV + st * C::kTileBytes;
+                    const uint32_t pcol = tmem + ((itg & 1) ? C::kColP1 : C::kColP0);
+#pragma unroll
+                    for (int ks = 0; ks < kBN / 16; ++ks) {
+                        const uint64_t bdesc = sdesc_sw128(vbase + ks * 2048, 16384, 1024);
+                        umma_bf16_ts(tmem + C::kColO, pcol + ks * 8, bdesc, idPV, (j > 0 || ks > 0) ? 1u : 0u);
+                    }
+                    umma_commit(smem_u32(&bar_p_free[itg & 1]));
+                    umma_commit(smem_u32(&bar_kv_empty[st]));  // K was read by S of this block, done before P
+                }
+                if (!ok) break;
+                kv_it += nblk;
+                s_it += nblk;
+            }
+            if (!ok) {
+                umma_commit(smem_u32(&bar_drain_pv));
+                mbar_wait_drain(smem_u32(&bar_drain_pv), 0);
+            }
+        }
+    } else if (warp < 6) {
         // ------------------------------------------------------------ softmax
         const int quad = warp & 3;  // TMEM lane quadrant this warp may access
         const int r = quad * 32 + lane;
@@ -557,7 +582,7 @@ int launch_fwd(const FwdParams& prm, int n_items_upper, cudaStream_t st)
         attr_done = true;
     }
     const int grid = max(1, min(n_items_upper, device_sm_count()));
-    attn_fwd_kernel<D, GLOBAL><<<grid, 192, C::kSmemBytes, st>>>(prm);
+    attn_fwd_kernel<D, GLOBAL><<<grid, 224, C::kSmemBytes, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
