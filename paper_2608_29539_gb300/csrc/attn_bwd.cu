@@ -459,7 +459,7 @@ struct Bwd2Cfg {
     static constexpr uint32_t kColDV = 128;
     static constexpr uint32_t kColBuf = 256;  // buffer b: S^T at 256+128b (64 cols), dP^T at +64
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr int kThreads = 480;
+    static constexpr int kThreads = 512;
 };
 
 template <bool GLOBAL>
@@ -500,6 +500,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t bar_kv_full, bar_kv_empty, bar_dkv_full, bar_dkv_empty, bar_drain, bar_stage;
+    __shared__ __align__(8) uint64_t bar_drain_b;
     __shared__ __align__(8) uint64_t bar_qdo_full[NS], bar_qdo_empty[NS];
     __shared__ __align__(8) uint64_t bar_st_full[2], bar_ds_full[2], bar_dq_full[2], bar_dq_empty[2];
     __shared__ uint32_t tmem_base_sh;
@@ -523,6 +524,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
         mbar_init(smem_u32(&bar_dkv_full), 1);
         mbar_init(smem_u32(&bar_dkv_empty), 128);
         mbar_init(smem_u32(&bar_drain), 1);
+        mbar_init(smem_u32(&bar_drain_b), 1);
         mbar_init(smem_u32(&bar_stage), 256);
         for (int s = 0; s < NS; ++s) {
             mbar_init(smem_u32(&bar_qdo_full[s]), 1);
@@ -589,39 +591,14 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+        // ------------------------------------------------------------ MMA issuer A: S^T, dP^T
+        // The tile's second half (dV, dK, dQ^T) comes from warp 15: two issuing
+        // threads keep the tensor pipe fed while either waits for its inputs
+        // (the issue queue is short, so one thread that stops to wait starves it).
         if (lane == 0) {
             constexpr uint32_t idS = idesc_bf16_f32(kBN, BQ, false, false);  // S^T, dP^T: 128 x 64
-            constexpr uint32_t idKV = idesc_bf16_f32(kBN, D, false, true);   // dV, dK: 128 x 128
-            constexpr uint32_t idQ = idesc_bf16_f32(D, BQ, true, true);      // dQ^T: 128 x 64
             int u = 0, kv_items = 0;
             bool ok = true;
-            // second half of tile v: dV, dK, dQ^T (x_in_item: position of v in its item)
-            auto issue_b = [&](int v, int x_in_item) -> bool {
-                const int b = v & 1, st = v % NS;
-                if (!mbar_wait(smem_u32(&bar_ds_full[b]), (v >> 1) & 1, &abort_flag)) return false;
-                if (x_in_item == 0 && !mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))
-                    return false;
-                tc_fence_after();
-                const uint32_t pb = sP + b * C::kPBytes, db = sDS + b * C::kPBytes;
-                const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
-#pragma unroll
-                for (int ks = 0; ks < BQ / 16; ++ks) {
-                    const uint32_t acc = (x_in_item > 0 || ks > 0) ? 1u : 0u;
-                    umma_bf16_ss(tmem + C::kColDV, sdesc_sw128(pb + ks * 32, 16, 1024),
-                                 sdesc_sw128(ob + ks * 2048, 8192, 1024), idKV, acc);
-                    umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
-                                 sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
-                }
-#pragma unroll
-                for (int ks = 0; ks < kBN / 16; ++ks) {
-                    umma_bf16_ss(tmem + C::kColBuf + 128 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
-                                 sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
-                }
-                umma_commit(smem_u32(&bar_dq_full[b]));
-                umma_commit(smem_u32(&bar_qdo_empty[st]));
-                return true;
-            };
             for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
                 const BwdItem it = decode_bwd2<GLOBAL>(p, k);
                 if (it.ntiles == 0) continue;
@@ -630,6 +607,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 for (int x = 0; x < n_it; ++x, ++u) {
                     const int b = u & 1, st = u % NS;
                     if (!(ok = mbar_wait(smem_u32(&bar_qdo_full[st]), (u / NS) & 1, &abort_flag))) break;
+                    // buffer b held dQ^T of tile u-2: the drain warps have read it
                     if (!(ok = mbar_wait(smem_u32(&bar_dq_empty[b]), ((u >> 1) & 1) ^ 1, &abort_flag))) break;
                     tc_fence_after();
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
@@ -649,17 +627,59 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                                      ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_st_full[b]));
-                    if (x > 0 && !(ok = issue_b(u - 1, x - 1))) break;
                 }
                 if (!ok) break;
-                if (!(ok = issue_b(u - 1, n_it - 1))) break;
-                umma_commit(smem_u32(&bar_kv_empty));
-                umma_commit(smem_u32(&bar_dkv_full));
                 ++kv_items;
             }
             if (!ok) {
                 umma_commit(smem_u32(&bar_drain));
                 mbar_wait_drain(smem_u32(&bar_drain), 0);
+            }
+        }
+    } else if (warp == 15) {
+        // ------------------------------------------------------------ MMA issuer B: dV, dK, dQ^T
+        if (lane == 0) {
+            constexpr uint32_t idKV = idesc_bf16_f32(kBN, D, false, true);  // dV, dK: 128 x 128
+            constexpr uint32_t idQ = idesc_bf16_f32(D, BQ, true, true);     // dQ^T: 128 x 64
+            int u = 0, kv_items = 0;
+            bool ok = true;
+            for (int k = blockIdx.x; k < n_items && ok; k += gridDim.x) {
+                const BwdItem it = decode_bwd2<GLOBAL>(p, k);
+                if (it.ntiles == 0) continue;
+                const int n_it = group * it.ntiles;
+                for (int x = 0; x < n_it; ++x, ++u) {
+                    const int b = u & 1, st = u % NS;
+                    if (!(ok = mbar_wait(smem_u32(&bar_ds_full[b]), (u >> 1) & 1, &abort_flag))) break;
+                    if (x == 0 && !(ok = mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))) break;
+                    tc_fence_after();
+                    const uint32_t pb = sP + b * C::kPBytes, db = sDS + b * C::kPBytes;
+                    const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
+#pragma unroll
+                    for (int ks = 0; ks < BQ / 16; ++ks) {
+                        const uint32_t acc = (x > 0 || ks > 0) ? 1u : 0u;
+                        umma_bf16_ss(tmem + C::kColDV, sdesc_sw128(pb + ks * 32, 16, 1024),
+                                     sdesc_sw128(ob + ks * 2048, 8192, 1024), idKV, acc);
+                        umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
+                                     sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
+                    }
+                    // dQ^T into the S^T columns of buffer b (read by the softmax before ds_full)
+#pragma unroll
+                    for (int ks = 0; ks < kBN / 16; ++ks) {
+                        umma_bf16_ss(tmem + C::kColBuf + 128 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
+                                     sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
+                    }
+                    umma_commit(smem_u32(&bar_dq_full[b]));
+                    umma_commit(smem_u32(&bar_qdo_empty[st]));
+                }
+                if (!ok) break;
+                // the item's last reads of K and V (S^T, dP^T of issuer A finished before ds_full)
+                umma_commit(smem_u32(&bar_kv_empty));
+                umma_commit(smem_u32(&bar_dkv_full));
+                ++kv_items;
+            }
+            if (!ok) {
+                umma_commit(smem_u32(&bar_drain_b));
+                mbar_wait_drain(smem_u32(&bar_drain_b), 0);
             }
         }
     } else if (warp < 10) {
