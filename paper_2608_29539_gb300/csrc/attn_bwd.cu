@@ -428,19 +428,21 @@ __global__ void __launch_bounds__(192, 1) attn_bwd_kernel(const __grid_constant_
 }
 
 // ---------------------------------------------------------------- d = 128
-// Overlapped variant for D = 128: query tiles of 64 rows with two TMEM
-// buffers, so the MMAs of tile u+1 (S^T, dP^T) run while the softmax warps
-// work on tile u, and dQ is produced transposed (dQ^T = K^T dS^T, one TMEM lane
-// per head-dim row) into the columns S^T of that tile occupied.  Roles:
+// Overlapped variant for D = 128: query tiles of 64 rows.  S^T and dP^T of a
+// tile share one TMEM buffer that the softmax warps release as soon as they
+// have loaded it, so the MMAs of tile u+1 run while the softmax works on tile
+// u; dQ is produced transposed (dQ^T = K^T dS^T, one TMEM lane per head-dim
+// row) into one of two buffers of its own.  Roles:
 //   warp 0       TMA: K/V per item, Q/dO tiles through a 3-deep ring
-//   warp 1       MMA issuer: S^T, dP^T (M=128 keys, N=64 queries) into buffer
-//                u%2; then, once P^T/dS^T of tile u-1 are in shared memory,
+//   warp 1       MMA issuer A: S^T, dP^T (M=128 keys, N=64 queries)
+//   warp 15      MMA issuer B: once P^T/dS^T of a tile are in shared memory,
 //                dV += P^T dO, dK += dS^T Q, dQ^T = K^T dS^T
 //   warps 2..9   two warpgroups, one per 32-query half of the tile; thread =
 //                key row: P^T and dS^T (bf16) from S^T and dP^T
 //   warps 10..13 dQ^T out of TMEM (thread = head-dim row), coalesced fp32
 //                atomics into the dQ accumulator (one 128-byte row segment per
 //                warp instruction); dK/dV epilogue at the end of each item
+//   warp 14      global branch: zero rows of the dense dQ for unselected tokens
 struct Bwd2Cfg {
     static constexpr int D = 128;
     static constexpr int kBQ = 64;                 // queries per tile
@@ -457,7 +459,8 @@ struct Bwd2Cfg {
     static constexpr int kSmemBytes = kOffDS + 2 * kPBytes + 1024;
     static constexpr uint32_t kColDK = 0;
     static constexpr uint32_t kColDV = 128;
-    static constexpr uint32_t kColBuf = 256;  // buffer b: S^T at 256+128b (64 cols), dP^T at +64
+    static constexpr uint32_t kColS = 256;    // S^T (64 cols), dP^T at +64
+    static constexpr uint32_t kColDQ = 384;   // dQ^T buffer b at 384 + 64b
     static constexpr uint32_t kTmemCols = 512;
     static constexpr int kThreads = 512;
 };
@@ -502,7 +505,8 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
     __shared__ __align__(8) uint64_t bar_kv_full, bar_kv_empty, bar_dkv_full, bar_dkv_empty, bar_drain, bar_stage;
     __shared__ __align__(8) uint64_t bar_drain_b;
     __shared__ __align__(8) uint64_t bar_qdo_full[NS], bar_qdo_empty[NS];
-    __shared__ __align__(8) uint64_t bar_st_full[2], bar_ds_full[2], bar_dq_full[2], bar_dq_empty[2];
+    __shared__ __align__(8) uint64_t bar_st_full, bar_st_empty;
+    __shared__ __align__(8) uint64_t bar_ds_full[2], bar_dq_full[2], bar_dq_empty[2];
     __shared__ uint32_t tmem_base_sh;
     __shared__ volatile int abort_flag;
     __shared__ int sh_pos[2][BQ];
@@ -530,8 +534,9 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             mbar_init(smem_u32(&bar_qdo_full[s]), 1);
             mbar_init(smem_u32(&bar_qdo_empty[s]), 1);
         }
+        mbar_init(smem_u32(&bar_st_full), 1);
+        mbar_init(smem_u32(&bar_st_empty), 256);
         for (int b = 0; b < 2; ++b) {
-            mbar_init(smem_u32(&bar_st_full[b]), 1);
             mbar_init(smem_u32(&bar_ds_full[b]), 256);
             mbar_init(smem_u32(&bar_dq_full[b]), 1);
             mbar_init(smem_u32(&bar_dq_empty[b]), 128);
@@ -605,13 +610,13 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 if (!(ok = mbar_wait(smem_u32(&bar_kv_full), kv_items & 1, &abort_flag))) break;
                 const int n_it = group * it.ntiles;
                 for (int x = 0; x < n_it; ++x, ++u) {
-                    const int b = u & 1, st = u % NS;
+                    const int st = u % NS;
                     if (!(ok = mbar_wait(smem_u32(&bar_qdo_full[st]), (u / NS) & 1, &abort_flag))) break;
-                    // buffer b held dQ^T of tile u-2: the drain warps have read it
-                    if (!(ok = mbar_wait(smem_u32(&bar_dq_empty[b]), ((u >> 1) & 1) ^ 1, &abort_flag))) break;
+                    // the softmax warps have loaded S^T, dP^T of tile u-1
+                    if (!(ok = mbar_wait(smem_u32(&bar_st_empty), (u & 1) ^ 1, &abort_flag))) break;
                     tc_fence_after();
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
-                    const uint32_t scol = tmem + C::kColBuf + 128 * b;
+                    const uint32_t scol = tmem + C::kColS;
 #pragma unroll
                     for (int ks = 0; ks < D / 16; ++ks) {
                         const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;
@@ -626,7 +631,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                         umma_bf16_ss(scol + 64, sdesc_sw128(sV + ka, 16, 1024), sdesc_sw128(ob + kb, 16, 1024), idS,
                                      ks > 0 ? 1u : 0u);
                     }
-                    umma_commit(smem_u32(&bar_st_full[b]));
+                    umma_commit(smem_u32(&bar_st_full));
                 }
                 if (!ok) break;
                 ++kv_items;
@@ -651,6 +656,8 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                     const int b = u & 1, st = u % NS;
                     if (!(ok = mbar_wait(smem_u32(&bar_ds_full[b]), (u >> 1) & 1, &abort_flag))) break;
                     if (x == 0 && !(ok = mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))) break;
+                    // dQ^T buffer b: the drain warps have read tile u-2's
+                    if (!(ok = mbar_wait(smem_u32(&bar_dq_empty[b]), ((u >> 1) & 1) ^ 1, &abort_flag))) break;
                     tc_fence_after();
                     const uint32_t pb = sP + b * C::kPBytes, db = sDS + b * C::kPBytes;
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
@@ -662,10 +669,9 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                         umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
                                      sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
                     }
-                    // dQ^T into the S^T columns of buffer b (read by the softmax before ds_full)
 #pragma unroll
                     for (int ks = 0; ks < kBN / 16; ++ks) {
-                        umma_bf16_ss(tmem + C::kColBuf + 128 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
+                        umma_bf16_ss(tmem + C::kColDQ + 64 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
                                      sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_dq_full[b]));
@@ -698,33 +704,32 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             const int k0 = it.j * kBN;
             const int key = k0 + t;
             const int n_it = group * it.ntiles;
-            // staging values of tile x (query positions, lse in log2 units,
-            // Dsum, "sees every key" flag): loaded one tile ahead so the global
-            // loads overlap the previous tile's work
+            // staging values of tile x (query position, lse, Dsum; -1 / 0 / 0
+            // outside the tile's rows): loaded one tile ahead and used only at
+            // the next tile, so no instruction waits for the loads while the
+            // current tile is computed
             int pf_pos = -1;
-            float2 pf_ld = make_float2(0.f, 0.f);
-            bool pf_open = false;
+            float pf_lse = 0.f, pf_dsum = 0.f;
             auto load_stage = [&](int x) {
                 const int h = it.kvh * group + x / it.ntiles;
                 const int i = it.i_lo + x % it.ntiles;
                 pf_pos = -1;
-                pf_ld = make_float2(0.f, 0.f);
-                pf_open = false;
+                pf_lse = pf_dsum = 0.f;
                 if (!GLOBAL) {
                     const int q = i * BQ + tw;
                     if (q < p.T) {
                         const int64_t idx = (static_cast<int64_t>(it.b) * p.Hq + h) * p.T + q;
                         pf_pos = q;
-                        pf_ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
-                        pf_open = q >= k0 + kBN - 1 && q - k0 < window;
+                        pf_lse = p.lse[idx];
+                        pf_dsum = p.dsum[idx];
                     }
                 } else {
                     const int row = i * BQ + tw;
                     if (row >= it.row_lo && row < it.row_hi) {
                         const int64_t idx = static_cast<int64_t>(h) * p.cap + row;
                         pf_pos = p.pos[row];
-                        pf_ld = make_float2(p.lse[idx] * kLog2e, p.dsum[idx]);
-                        pf_open = pf_pos >= k0 + kBN - 1;
+                        pf_lse = p.lse[idx];
+                        pf_dsum = p.dsum[idx];
                     }
                 }
             };
@@ -732,10 +737,12 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             for (int x = 0; x < n_it; ++x, ++u) {
                 const int b = u & 1;
                 if (tw < BQ) {
+                    // lse in log2 units; "sees every key of the block"
+                    const bool pf_open = pf_pos >= k0 + kBN - 1 && (GLOBAL || pf_pos - k0 < window);
                     sh_pos[b][tw] = pf_pos;
                     float* pr = reinterpret_cast<float*>(&sh_pair[b][tw >> 1]);
-                    pr[tw & 1] = -pf_ld.x;
-                    pr[2 + (tw & 1)] = -pf_ld.y;
+                    pr[tw & 1] = -(pf_lse * kLog2e);
+                    pr[2 + (tw & 1)] = -pf_dsum;
                     const bool all_open = __all_sync(0xffffffffu, pf_open);
                     if (lane == 0) sh_open[b][tw >> 5] = all_open ? 1 : 0;
                 }
@@ -744,7 +751,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 if (!ok) break;
                 if (tw < BQ && x + 1 < n_it) load_stage(x + 1);
                 const bool open = sh_open[b][0] && sh_open[b][1];
-                ok = mbar_wait(smem_u32(&bar_st_full[b]), (u >> 1) & 1, &abort_flag);
+                ok = mbar_wait(smem_u32(&bar_st_full), u & 1, &abort_flag);
                 __syncwarp();
                 if (!ok) break;
                 // P^T / dS^T buffer b is free once the MMAs of tile u-2 are done
@@ -754,9 +761,11 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 if (!ok) break;
                 tc_fence_after();
                 uint32_t sv[32], dpv[32];
-                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + half * 32, sv);
-                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + 64 + half * 32, dpv);
+                tmem_ld32(tmem + lane_off + C::kColS + half * 32, sv);
+                tmem_ld32(tmem + lane_off + C::kColS + 64 + half * 32, dpv);
                 tmem_wait_ld();
+                tc_fence_before();
+                mbar_arrive(smem_u32(&bar_st_empty));  // S^T, dP^T of tile u+1 may now be written
                 uint32_t pk[16], dk2[16];
                 // P = 2^(S*scale*log2e - lse), dS = P (dP - Dsum), two columns per
                 // f32x2 instruction.  Two branch-free copies of the loop (open
@@ -830,8 +839,8 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 if (!ok) break;
                 tc_fence_after();
                 uint32_t v0[32], v1[32];
-                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b, v0);
-                tmem_ld32(tmem + lane_off + C::kColBuf + 128 * b + 32, v1);
+                tmem_ld32(tmem + lane_off + C::kColDQ + 64 * b, v0);
+                tmem_ld32(tmem + lane_off + C::kColDQ + 64 * b + 32, v1);
                 tmem_wait_ld();
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_dq_empty[b]));
