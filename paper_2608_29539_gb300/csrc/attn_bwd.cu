@@ -431,9 +431,10 @@ __global__ void __launch_bounds__(192, 1) attn_bwd_kernel(const __grid_constant_
 // Overlapped variant for D = 128: query tiles of 64 rows.  S^T and dP^T of a
 // tile share one TMEM buffer that the softmax warps release as soon as they
 // have loaded it, so the MMAs of tile u+1 run while the softmax works on tile
-// u; dQ is produced transposed (dQ^T = K^T dS^T, one TMEM lane per head-dim
-// row) into one of two buffers of its own.  Roles:
-//   warp 0       TMA: K/V per item, Q/dO tiles through a 3-deep ring
+// u.  P^T goes back to TMEM (two buffers; dV reads it as the TMEM operand),
+// dS^T to shared memory (two buffers; dK and dQ^T read it), and dQ is produced
+// transposed (dQ^T = K^T dS^T, one TMEM lane per head-dim row).  Roles:
+//   warp 0       TMA: K/V per item, Q/dO tiles through a 4-deep ring
 //   warp 1       MMA issuer A: S^T, dP^T (M=128 keys, N=64 queries)
 //   warp 15      MMA issuer B: once P^T/dS^T of a tile are in shared memory,
 //                dV += P^T dO, dK += dS^T Q, dQ^T = K^T dS^T
@@ -446,21 +447,21 @@ __global__ void __launch_bounds__(192, 1) attn_bwd_kernel(const __grid_constant_
 struct Bwd2Cfg {
     static constexpr int D = 128;
     static constexpr int kBQ = 64;                 // queries per tile
-    static constexpr int kStages = 3;              // Q/dO ring depth
+    static constexpr int kStages = 4;              // Q/dO ring depth
     static constexpr int kKVBytes = kBN * D * 2;   // K or V block: 32 KB
     static constexpr int kQBytes = kBQ * D * 2;    // Q or dO tile: 16 KB (two 8 KB halves of d)
-    static constexpr int kPBytes = kBN * kBQ * 2;  // P^T or dS^T: 16 KB
+    static constexpr int kPBytes = kBN * kBQ * 2;  // dS^T: 16 KB
     static constexpr int kOffK = 0;
     static constexpr int kOffV = kOffK + kKVBytes;
     static constexpr int kOffQ = kOffV + kKVBytes;
     static constexpr int kOffDO = kOffQ + kStages * kQBytes;
-    static constexpr int kOffP = kOffDO + kStages * kQBytes;  // 2 buffers
-    static constexpr int kOffDS = kOffP + 2 * kPBytes;        // 2 buffers
+    static constexpr int kOffDS = kOffDO + kStages * kQBytes;  // 2 buffers
     static constexpr int kSmemBytes = kOffDS + 2 * kPBytes + 1024;
     static constexpr uint32_t kColDK = 0;
     static constexpr uint32_t kColDV = 128;
     static constexpr uint32_t kColS = 256;    // S^T (64 cols), dP^T at +64
-    static constexpr uint32_t kColDQ = 384;   // dQ^T buffer b at 384 + 64b
+    static constexpr uint32_t kColDQ = 384;   // dQ^T (64 cols)
+    static constexpr uint32_t kColP = 448;    // P^T buffer b (bf16 pairs) at 448 + 32b
     static constexpr uint32_t kTmemCols = 512;
     static constexpr int kThreads = 512;
 };
@@ -517,7 +518,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t sK = smem_u32(smem + C::kOffK), sV = smem_u32(smem + C::kOffV);
     const uint32_t sQ = smem_u32(smem + C::kOffQ), sDO = smem_u32(smem + C::kOffDO);
-    const uint32_t sP = smem_u32(smem + C::kOffP), sDS = smem_u32(smem + C::kOffDS);
+    const uint32_t sDS = smem_u32(smem + C::kOffDS);
     const int group = p.Hq / p.Hkv;
     const int n_items = p.B * p.nblk * p.Hkv;
 
@@ -656,22 +657,23 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                     const int b = u & 1, st = u % NS;
                     if (!(ok = mbar_wait(smem_u32(&bar_ds_full[b]), (u >> 1) & 1, &abort_flag))) break;
                     if (x == 0 && !(ok = mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))) break;
-                    // dQ^T buffer b: the drain warps have read tile u-2's
-                    if (!(ok = mbar_wait(smem_u32(&bar_dq_empty[b]), ((u >> 1) & 1) ^ 1, &abort_flag))) break;
+                    // dQ^T: the drain warps have read tile u-1's
+                    if (u > 0 && !(ok = mbar_wait(smem_u32(&bar_dq_empty[b ^ 1]), ((u - 1) >> 1) & 1, &abort_flag)))
+                        break;
                     tc_fence_after();
-                    const uint32_t pb = sP + b * C::kPBytes, db = sDS + b * C::kPBytes;
+                    const uint32_t db = sDS + b * C::kPBytes;
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
 #pragma unroll
                     for (int ks = 0; ks < BQ / 16; ++ks) {
                         const uint32_t acc = (x > 0 || ks > 0) ? 1u : 0u;
-                        umma_bf16_ss(tmem + C::kColDV, sdesc_sw128(pb + ks * 32, 16, 1024),
+                        umma_bf16_ts(tmem + C::kColDV, tmem + C::kColP + 32 * b + 8 * ks,
                                      sdesc_sw128(ob + ks * 2048, 8192, 1024), idKV, acc);
                         umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
                                      sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
                     }
 #pragma unroll
                     for (int ks = 0; ks < kBN / 16; ++ks) {
-                        umma_bf16_ss(tmem + C::kColDQ + 64 * b, sdesc_sw128(sK + ks * 2048, 16384, 1024),
+                        umma_bf16_ss(tmem + C::kColDQ, sdesc_sw128(sK + ks * 2048, 16384, 1024),
                                      sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_dq_full[b]));
@@ -754,7 +756,7 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 ok = mbar_wait(smem_u32(&bar_st_full), u & 1, &abort_flag);
                 __syncwarp();
                 if (!ok) break;
-                // P^T / dS^T buffer b is free once the MMAs of tile u-2 are done
+                // P^T (TMEM) / dS^T (shared) buffer b is free once the MMAs of tile u-2 are done
                 // (they were issued before S^T of tile u, so this rarely waits)
                 ok = mbar_wait(smem_u32(&bar_dq_full[b]), ((u >> 1) & 1) ^ 1, &abort_flag);
                 __syncwarp();
@@ -797,13 +799,16 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 };
                 if (open) columns(std::false_type{});
                 else columns(std::true_type{});
+                // P^T row t: query columns half*32.. as 16 bf16 pairs, the TMEM
+                // operand layout (column c holds queries 2c, 2c+1)
+                tmem_st16(tmem + lane_off + C::kColP + 32 * b + half * 16, pk);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     const uint32_t off = sw128_offset(t, half * 4 + q4);
-                    st_shared_v4(sP + b * C::kPBytes + off, pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
                     st_shared_v4(sDS + b * C::kPBytes + off, dk2[4 * q4], dk2[4 * q4 + 1], dk2[4 * q4 + 2],
                                  dk2[4 * q4 + 3]);
                 }
+                tmem_wait_st();
                 fence_proxy_async_smem();
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_ds_full[b]));
@@ -839,8 +844,8 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 if (!ok) break;
                 tc_fence_after();
                 uint32_t v0[32], v1[32];
-                tmem_ld32(tmem + lane_off + C::kColDQ + 64 * b, v0);
-                tmem_ld32(tmem + lane_off + C::kColDQ + 64 * b + 32, v1);
+                tmem_ld32(tmem + lane_off + C::kColDQ, v0);
+                tmem_ld32(tmem + lane_off + C::kColDQ + 32, v1);
                 tmem_wait_ld();
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_dq_empty[b]));
