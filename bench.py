@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "abb0191c1d6121c0"): 824374784 + 479653888,
-    ("global_bwd", "abb0191c1d6121c0"): 463391488 + 427855104,
+    ("local_bwd", "a9e31f5a2c17cf68"): 823936000 + 479489280,
+    ("global_bwd", "a9e31f5a2c17cf68"): 471555840 + 433355008,
 }
 
 
