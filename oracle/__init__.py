@@ -80,6 +80,8 @@ def _load():
             lib.oracle_combine_bwd.argtypes = [_f32p, _f32p, _f32p, _f32p, _u8p, _i32p, ctypes.c_void_p,
                                                ctypes.c_void_p, ctypes.c_double, _int, _int, _int, _int,
                                                _f64p, _f64p, _f64p]
+            lib.oracle_combine_dgain.argtypes = [_f32p, _f32p, _f32p, _f32p, _u8p, _i32p, ctypes.c_double,
+                                                 _int, _int, _int, _int, _f64p, _f64p]
             lib.oracle_num_threads.restype = _int
             _lib = lib
     return _lib
@@ -257,3 +259,18 @@ def combine_bwd(dO, oL, oGc, p, z, row_of, gL=None, gG=None, eps: float = 1e-6):
     _load().oracle_combine_bwd(_f32(dO), oL, oGc, _f32(p), np.ascontiguousarray(z, dtype=np.uint8),
                                _i32(row_of), gL_p, gG_p, float(eps), B, T, H, D, dOL, dOG, dp)
     return dOL, dOG[:n], dp
+
+
+def combine_dgain(dO, oL, oGc, p, z, row_of, eps: float = 1e-6):
+    """Gradients of the ContextNorm gains of Eq. 9 with z fixed: (dgL, dgG),
+    each [H, D] float64 (the gains' own values do not enter: o~ is linear in
+    them)."""
+    oL = _f32(oL)
+    B, T, H, D = oL.shape
+    n = int(np.asarray(z).sum())
+    oGc = _f32(oGc).reshape(-1, H, D) if n else np.zeros((1, H, D), np.float32)
+    dgL = np.zeros((H, D), dtype=np.float64)
+    dgG = np.zeros((H, D), dtype=np.float64)
+    _load().oracle_combine_dgain(_f32(dO), oL, oGc, _f32(p), np.ascontiguousarray(z, dtype=np.uint8),
+                                 _i32(row_of), float(eps), B, T, H, D, dgL, dgG)
+    return dgL, dgG

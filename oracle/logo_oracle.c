@@ -348,6 +348,40 @@ void oracle_combine_bwd(const float* dO, const float* oL, const float* oGc, cons
     }
 }
 
+/* Gradients of the ContextNorm gains (Eq. 9, o~ = o * r * gain per head and
+ * dimension) with z fixed as in oracle_combine_bwd.  o~ is linear in the gain,
+ * so with dy the gradient reaching o~ (dy^L = dO (1 - p z), dy^G = dO p):
+ *   dgL[h,d] = sum over every token of dy^L_d * oL_d * r^L
+ *   dgG[h,d] = sum over the selected tokens of dy^G_d * oG_d * r^G
+ * Summed in double over the tokens in order (b, t), serially. */
+void oracle_combine_dgain(const float* dO, const float* oL, const float* oGc, const float* p,
+                          const uint8_t* z, const int32_t* row_of, double eps, int B, int T, int H, int D,
+                          double* dgL, double* dgG)
+{
+    int64_t ntok = (int64_t)B * T;
+    memset(dgL, 0, sizeof(double) * (size_t)H * (size_t)D);
+    memset(dgG, 0, sizeof(double) * (size_t)H * (size_t)D);
+    for (int64_t bt = 0; bt < ntok; ++bt) {
+        double pt = (double)p[bt];
+        double wl = z[bt] ? 1.0 - pt : 1.0;
+        for (int h = 0; h < H; ++h) {
+            const float* g = dO + (bt * H + h) * (int64_t)D;
+            const float* xl = oL + (bt * H + h) * (int64_t)D;
+            double ss = 0.0;
+            for (int d = 0; d < D; ++d) ss += (double)xl[d] * (double)xl[d];
+            double rl = 1.0 / sqrt(ss / D + eps);
+            for (int d = 0; d < D; ++d) dgL[(int64_t)h * D + d] += (double)g[d] * wl * (double)xl[d] * rl;
+            if (z[bt]) {
+                const float* xg = oGc + ((int64_t)row_of[bt] * H + h) * (int64_t)D;
+                double sg = 0.0;
+                for (int d = 0; d < D; ++d) sg += (double)xg[d] * (double)xg[d];
+                double rg = 1.0 / sqrt(sg / D + eps);
+                for (int d = 0; d < D; ++d) dgG[(int64_t)h * D + d] += (double)g[d] * pt * (double)xg[d] * rg;
+            }
+        }
+    }
+}
+
 int oracle_num_threads(void)
 {
 #ifdef _OPENMP

@@ -434,6 +434,54 @@ def test_combine_bwd_matches_torch_autograd():
     np.testing.assert_allclose(dp, tp.grad.numpy(), rtol=1e-9, atol=1e-12)
 
 
+def test_gain_grads_match_torch_autograd():
+    oL, oGc, p, z, row_of, gL, gG, n = _setup_combine()
+    dO = _rand(*oL.shape)
+    dgL, dgG = oracle.combine_dgain(dO, oL, oGc, p, z, row_of)
+    B, T, H, D = oL.shape
+    wL = torch.tensor(gL, dtype=torch.float64, requires_grad=True)
+    wG = torch.tensor(gG, dtype=torch.float64, requires_grad=True)
+    nL = torch.stack([F.rms_norm(torch.tensor(oL[:, :, h], dtype=torch.float64), (D,), weight=wL[h], eps=1e-6)
+                      for h in range(H)], dim=2)
+    nG = torch.stack([F.rms_norm(torch.tensor(oGc[:, h], dtype=torch.float64), (D,), weight=wG[h], eps=1e-6)
+                      for h in range(H)], dim=1)
+    bb, tt = np.nonzero(z)
+    full_g = torch.zeros_like(nL).index_put((torch.tensor(bb), torch.tensor(tt)), nG)
+    zt = torch.tensor(z, dtype=torch.float64)[..., None, None]
+    pp = torch.tensor(p, dtype=torch.float64)[..., None, None]
+    o = zt * ((1 - pp) * nL + pp * full_g) + (1 - zt) * nL
+    o.backward(torch.tensor(dO, dtype=torch.float64))
+    np.testing.assert_allclose(dgL, wL.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(dgG, wG.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_gain_grads_finite_differences_and_special_cases():
+    oL, oGc, p, z, row_of, gL, gG, n = _setup_combine(B=1, T=7, H=2, D=8, ratio_k=3)
+    dO = _rand(*oL.shape)
+    dgL, dgG = oracle.combine_dgain(dO, oL, oGc, p, z, row_of)
+
+    def loss(gL_, gG_):
+        o, _, _ = oracle.combine_fwd(oL, oGc, p, z, row_of, gL_, gG_)
+        return float((o * dO.astype(np.float64)).sum())
+
+    for idx in [(0, 0), (1, 5), (0, 7)]:
+        for which in (0, 1):
+            hi = [gL.copy(), gG.copy()]
+            lo = [gL.copy(), gG.copy()]
+            hi[which][idx] += np.float32(0.25)
+            lo[which][idx] -= np.float32(0.25)
+            step = float(hi[which][idx]) - float(lo[which][idx])
+            fd = (loss(*hi) - loss(*lo)) / step  # exact up to rounding: the output is linear in a gain
+            assert fd == pytest.approx((dgL, dgG)[which][idx], rel=1e-9, abs=1e-12)
+    # nothing selected: no gradient reaches the global gain; p = 0 on the selected
+    # tokens: the local gain sees dO itself on every token
+    dgL0, dgG0 = oracle.combine_dgain(dO, oL, oGc, p, np.zeros_like(z), row_of)
+    assert (dgG0 == 0).all()
+    _, rL, _ = oracle.combine_fwd(oL, oGc, p, np.zeros_like(z), row_of, None, None)
+    ref = (dO.astype(np.float64) * oL.astype(np.float64) * rL[..., None]).sum(axis=(0, 1))
+    np.testing.assert_allclose(dgL0, ref, rtol=1e-12, atol=1e-12)
+
+
 def test_ratio_zero_layer_is_pure_local():
     # rho = 0: no token is selected, the layer output is Norm^L(O^L) and no
     # gradient reaches the global branch or the gate.
