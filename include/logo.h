@@ -269,7 +269,9 @@ LOGO_API int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* k,
  *      [B,T] float32; z [B,T] uint8; row_of [B,T] int32; gain_l / gain_g
  *      [Hq,D] float32 or NULL (= 1); eps > 0.
  * Out: o [B,T,Hq,D] bf16; rstd_l [B,T,Hq] and rstd_g [B*T,Hq] float32 (the
- *      RMS reciprocals r; either may be NULL). */
+ *      RMS reciprocals r; either may be NULL).
+ * Errors: LOGO_ERR_UNSUPPORTED if D is not 64 or 128, Hq*D > 16384, or a
+ *      bf16 / gain pointer is not 16-byte aligned. */
 LOGO_API int logo_combine(const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p, const uint8_t* z,
                  const int32_t* row_of, const float* gain_l, const float* gain_g, float eps, logo_bf16* o,
                  float* rstd_l, float* rstd_g, logo_dims dims, void* stream);
@@ -283,6 +285,23 @@ LOGO_API int logo_combine(const logo_bf16* o_l, const logo_bf16* o_c, const floa
 LOGO_API int logo_combine_bwd(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p,
                      const uint8_t* z, const int32_t* row_of, const float* gain_l, const float* gain_g, float eps,
                      logo_bf16* dO_l, logo_bf16* dO_c, float* dgate_p, logo_dims dims, void* stream);
+
+/* logo_combine_bwd_gains -- logo_combine_bwd plus the gradients of the two
+ *   ContextNorm gains (Eq. 9; o~ = o r gain is linear in the gain), z fixed:
+ *   dgain_l[h,d] = sum over every token of dy^L o^L r^L, dy^L = dO (1 - p z);
+ *   dgain_g[h,d] = sum over the selected tokens of dy^G o^G r^G, dy^G = dO p.
+ * Out: as logo_combine_bwd, plus dgain_l / dgain_g [Hq,D] float32 (overwritten;
+ *      either may be NULL, not both).  Tokens are summed per block, then the
+ *      blocks in a fixed order: the result is deterministic on a given GPU.
+ * Workspace: logo_combine_bwd_workspace_size(dims) bytes of device memory.
+ * Errors: LOGO_ERR_UNSUPPORTED if Hq*D > 8192; LOGO_ERR_WORKSPACE if the
+ *      workspace is short; otherwise as logo_combine_bwd. */
+LOGO_API size_t logo_combine_bwd_workspace_size(logo_dims dims);
+LOGO_API int logo_combine_bwd_gains(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c,
+                                    const float* gate_p, const uint8_t* z, const int32_t* row_of,
+                                    const float* gain_l, const float* gain_g, float eps, logo_bf16* dO_l,
+                                    logo_bf16* dO_c, float* dgate_p, float* dgain_l, float* dgain_g,
+                                    logo_dims dims, void* workspace, size_t workspace_bytes, void* stream);
 
 #ifdef __cplusplus
 }

@@ -1,11 +1,16 @@
-// combine.cu -- logo_combine / logo_combine_bwd: ContextNorm (Eq. 9, a
-// head-wise RMSNorm over D per branch) fused with the gate-weighted output
-// fusion of Eq. 10, and the backward of both with z held fixed.
+// combine.cu -- logo_combine / logo_combine_bwd(_gains): ContextNorm (Eq. 9,
+// a head-wise RMSNorm over D per branch) fused with the gate-weighted output
+// fusion of Eq. 10, the backward of both with z held fixed, and the gradients
+// of the two ContextNorm gains.
 //
-// HBM-bound: one block per token; every thread owns 16-byte vectors (8 bf16)
-// of one head, the D/8 threads of a head reduce their sums with warp
-// shuffles, and the backward reduces dp_t over all heads of the token in
-// shared memory.  All arithmetic is fp32; inputs and outputs bf16.
+// HBM-bound.  Blocks walk the tokens (grid-stride); a thread owns VPT fixed
+// 16-byte vectors (8 bf16) of the token's [H, D] row, issues all of a token's
+// loads before any arithmetic (so each thread keeps VPT to 3*VPT loads in
+// flight), and the D/8 lanes of a head reduce their sums with warp shuffles.
+// The backward sums dp_t over every head of the token in shared memory, and
+// the gain gradients over tokens in registers (fixed vectors per thread), then
+// per block into a workspace that a second kernel reduces in block order
+// (deterministic).  All arithmetic is fp32; inputs and outputs bf16.
 #include <cuda_bf16.h>
 
 #include <cstdint>
@@ -16,15 +21,18 @@
 namespace logo {
 namespace {
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;
+constexpr int kMaxVec = 8 * kThreads;   // H*D/8 vectors per token at most (VPT <= 8)
+constexpr int kMaxVecGains = 4 * kThreads;
 
 struct Vec8 {
     float v[8];
 };
 
-__device__ __forceinline__ Vec8 load_bf16x8(const logo_bf16* p)
+__device__ __forceinline__ uint4 ld_vec(const logo_bf16* p) { return *reinterpret_cast<const uint4*>(p); }
+
+__device__ __forceinline__ Vec8 unpack8(const uint4& raw)
 {
-    uint4 raw = *reinterpret_cast<const uint4*>(p);
     Vec8 r;
     const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&raw);
 #pragma unroll
@@ -67,124 +75,228 @@ __device__ __forceinline__ float head_sum(float x, int width)
     return x;
 }
 
+template <int VPT>
 __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
     const logo_bf16* __restrict__ o_l, const logo_bf16* __restrict__ o_c, const float* __restrict__ gate_p,
     const uint8_t* __restrict__ z, const int32_t* __restrict__ row_of, const float* __restrict__ gain_l,
     const float* __restrict__ gain_g, float eps, logo_bf16* __restrict__ o, float* __restrict__ rstd_l,
-    float* __restrict__ rstd_g, int H, int D)
+    float* __restrict__ rstd_g, int64_t ntok, int H, int D)
 {
-    const int64_t bt = blockIdx.x;
     const int vpr = D / 8;               // vectors per head row
     const int nvec = H * vpr;            // vectors per token
-    const bool sel = z[bt] != 0;
-    const int64_t row = sel ? row_of[bt] : -1;
-    const float pt = gate_p[bt];
     const float inv_d = 1.0f / static_cast<float>(D);
-    for (int v0 = 0; v0 < nvec; v0 += kThreads) {
-        const int v = v0 + threadIdx.x;
-        const bool active = v < nvec;
-        const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
-        Vec8 xl = active ? load_bf16x8(o_l + (bt * H + h) * D + j * 8) : Vec8{};
-        float ss = 0.f;
+    for (int64_t bt = blockIdx.x; bt < ntok; bt += gridDim.x) {
+        const bool sel = z[bt] != 0;
+        const int64_t row = sel ? row_of[bt] : 0;
+        const float pt = gate_p[bt];
+        uint4 rl[VPT], rg[VPT];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) ss += xl.v[i] * xl.v[i];
-        ss = head_sum(ss, vpr);
-        const float rl = rsqrtf(ss * inv_d + eps);
-        Vec8 gl = load_gain(gain_l, h, D, j);
-        Vec8 out;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) out.v[i] = xl.v[i] * rl * gl.v[i];
-        float rg = 0.f;
-        if (sel) {
-            Vec8 xg = active ? load_bf16x8(o_c + (row * H + h) * D + j * 8) : Vec8{};
-            float sg = 0.f;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) sg += xg.v[i] * xg.v[i];
-            sg = head_sum(sg, vpr);
-            rg = rsqrtf(sg * inv_d + eps);
-            Vec8 gg = load_gain(gain_g, h, D, j);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) out.v[i] = (1.0f - pt) * out.v[i] + pt * (xg.v[i] * rg * gg.v[i]);
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            rl[k] = v < nvec ? ld_vec(o_l + (bt * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
+            rg[k] = (sel && v < nvec) ? ld_vec(o_c + (row * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
         }
-        if (active) {
-            store_bf16x8(o + (bt * H + h) * D + j * 8, out);
-            if (j == 0) {
-                if (rstd_l) rstd_l[bt * H + h] = rl;
-                if (sel && rstd_g) rstd_g[row * H + h] = rg;
+#pragma unroll
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            const bool active = v < nvec;
+            const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
+            const Vec8 xl = unpack8(rl[k]);
+            float ss = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) ss += xl.v[i] * xl.v[i];
+            ss = head_sum(ss, vpr);
+            const float r_l = rsqrtf(ss * inv_d + eps);
+            const Vec8 gl = load_gain(gain_l, h, D, j);
+            Vec8 out;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) out.v[i] = xl.v[i] * r_l * gl.v[i];
+            float r_g = 0.f;
+            if (sel) {
+                const Vec8 xg = unpack8(rg[k]);
+                float sg = 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) sg += xg.v[i] * xg.v[i];
+                sg = head_sum(sg, vpr);
+                r_g = rsqrtf(sg * inv_d + eps);
+                const Vec8 gg = load_gain(gain_g, h, D, j);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) out.v[i] = (1.0f - pt) * out.v[i] + pt * (xg.v[i] * r_g * gg.v[i]);
+            }
+            if (active) {
+                store_bf16x8(o + (bt * nvec + v) * 8, out);
+                if (j == 0) {
+                    if (rstd_l) rstd_l[bt * H + h] = r_l;
+                    if (sel && rstd_g) rstd_g[row * H + h] = r_g;
+                }
             }
         }
     }
 }
 
+// part (DGAIN): [gridDim.x][2][H*D] float32 per-block sums of the local and
+// global gain gradients.
+template <int VPT, bool DGAIN>
 __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     const logo_bf16* __restrict__ dO, const logo_bf16* __restrict__ o_l, const logo_bf16* __restrict__ o_c,
     const float* __restrict__ gate_p, const uint8_t* __restrict__ z, const int32_t* __restrict__ row_of,
     const float* __restrict__ gain_l, const float* __restrict__ gain_g, float eps, logo_bf16* __restrict__ dO_l,
-    logo_bf16* __restrict__ dO_c, float* __restrict__ dgate_p, int H, int D)
+    logo_bf16* __restrict__ dO_c, float* __restrict__ dgate_p, float* __restrict__ part, int64_t ntok, int H, int D)
 {
-    __shared__ float sh_dp[kThreads / 32];
-    const int64_t bt = blockIdx.x;
+    __shared__ float sh_dp[2][kThreads / 32];
     const int vpr = D / 8;
     const int nvec = H * vpr;
-    const bool sel = z[bt] != 0;
-    const int64_t row = sel ? row_of[bt] : -1;
-    const float pt = gate_p[bt];
-    const float wl = sel ? 1.0f - pt : 1.0f;
     const float inv_d = 1.0f / static_cast<float>(D);
-    float dp_acc = 0.f;
-    for (int v0 = 0; v0 < nvec; v0 += kThreads) {
-        const int v = v0 + threadIdx.x;
-        const bool active = v < nvec;
-        const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
-        Vec8 g = active ? load_bf16x8(dO + (bt * H + h) * D + j * 8) : Vec8{};
-        Vec8 xl = active ? load_bf16x8(o_l + (bt * H + h) * D + j * 8) : Vec8{};
-        Vec8 gl = load_gain(gain_l, h, D, j);
-        // local branch: dy = dO * wl; dx = r g dy - x r^3 mean(x g dy)
-        float ss = 0.f, xgdy = 0.f;
+    float accL[DGAIN ? VPT : 1][8], accG[DGAIN ? VPT : 1][8];
+    if (DGAIN) {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            ss += xl.v[i] * xl.v[i];
-            xgdy += xl.v[i] * gl.v[i] * g.v[i];
+        for (int k = 0; k < VPT; ++k)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) accL[k][i] = accG[k][i] = 0.f;
+    }
+    int n_sel_seen = 0;
+    for (int64_t bt = blockIdx.x; bt < ntok; bt += gridDim.x) {
+        const bool sel = z[bt] != 0;
+        const int64_t row = sel ? row_of[bt] : 0;
+        const float pt = gate_p[bt];
+        const float wl = sel ? 1.0f - pt : 1.0f;
+        uint4 rd[VPT], rl[VPT], rg[VPT];
+#pragma unroll
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            const bool active = v < nvec;
+            rd[k] = active ? ld_vec(dO + (bt * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
+            rl[k] = active ? ld_vec(o_l + (bt * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
+            rg[k] = (sel && active) ? ld_vec(o_c + (row * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
         }
-        ss = head_sum(ss, vpr);
-        xgdy = head_sum(xgdy, vpr) * wl;
-        const float rl = rsqrtf(ss * inv_d + eps);
-        const float cl = rl * rl * rl * xgdy * inv_d;
-        Vec8 dxl;
+        float dp_acc = 0.f;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) dxl.v[i] = rl * gl.v[i] * g.v[i] * wl - xl.v[i] * cl;
-        if (active) store_bf16x8(dO_l + (bt * H + h) * D + j * 8, dxl);
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            const bool active = v < nvec;
+            const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
+            const Vec8 g = unpack8(rd[k]);
+            const Vec8 xl = unpack8(rl[k]);
+            const Vec8 gl = load_gain(gain_l, h, D, j);
+            // local branch: dy = dO * wl; dx = r g dy - x r^3 mean(x g dy)
+            float ss = 0.f, xgdy = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                ss += xl.v[i] * xl.v[i];
+                xgdy += xl.v[i] * gl.v[i] * g.v[i];
+            }
+            ss = head_sum(ss, vpr);
+            xgdy = head_sum(xgdy, vpr) * wl;
+            const float r_l = rsqrtf(ss * inv_d + eps);
+            const float cl = r_l * r_l * r_l * xgdy * inv_d;
+            Vec8 dxl;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) dxl.v[i] = r_l * gl.v[i] * g.v[i] * wl - xl.v[i] * cl;
+            if (active) store_bf16x8(dO_l + (bt * nvec + v) * 8, dxl);
+            if (DGAIN) {  // d gain_l = dy * x r
+#pragma unroll
+                for (int i = 0; i < 8; ++i) accL[k][i] += g.v[i] * wl * xl.v[i] * r_l;
+            }
+            if (sel) {
+                const Vec8 xg = unpack8(rg[k]);
+                const Vec8 gg = load_gain(gain_g, h, D, j);
+                float sg = 0.f, xgdyg = 0.f;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    sg += xg.v[i] * xg.v[i];
+                    xgdyg += xg.v[i] * gg.v[i] * g.v[i];
+                }
+                sg = head_sum(sg, vpr);
+                xgdyg = head_sum(xgdyg, vpr) * pt;
+                const float r_g = rsqrtf(sg * inv_d + eps);
+                const float cg = r_g * r_g * r_g * xgdyg * inv_d;
+                Vec8 dxg;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    dxg.v[i] = r_g * gg.v[i] * g.v[i] * pt - xg.v[i] * cg;
+                    dp_acc += g.v[i] * (xg.v[i] * r_g * gg.v[i] - xl.v[i] * r_l * gl.v[i]);
+                }
+                if (active) store_bf16x8(dO_c + (row * nvec + v) * 8, dxg);
+                if (DGAIN) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) accG[k][i] += g.v[i] * pt * xg.v[i] * r_g;
+                }
+            }
+        }
+        // dp_t = z_t * sum_{h,d} dO (o~G - o~L); z_t is uniform over the block
         if (sel) {
-            Vec8 xg = active ? load_bf16x8(o_c + (row * H + h) * D + j * 8) : Vec8{};
-            Vec8 gg = load_gain(gain_g, h, D, j);
-            float sg = 0.f, xgdyg = 0.f;
+            const int buf = n_sel_seen & 1;
+            ++n_sel_seen;
+            dp_acc = head_sum(dp_acc, 32);
+            if ((threadIdx.x & 31) == 0) sh_dp[buf][threadIdx.x >> 5] = dp_acc;
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                float s = 0.f;
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                sg += xg.v[i] * xg.v[i];
-                xgdyg += xg.v[i] * gg.v[i] * g.v[i];
+                for (int w = 0; w < kThreads / 32; ++w) s += sh_dp[buf][w];
+                dgate_p[bt] = s;
             }
-            sg = head_sum(sg, vpr);
-            xgdyg = head_sum(xgdyg, vpr) * pt;
-            const float rg = rsqrtf(sg * inv_d + eps);
-            const float cg = rg * rg * rg * xgdyg * inv_d;
-            Vec8 dxg;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                dxg.v[i] = rg * gg.v[i] * g.v[i] * pt - xg.v[i] * cg;
-                dp_acc += g.v[i] * (xg.v[i] * rg * gg.v[i] - xl.v[i] * rl * gl.v[i]);
-            }
-            if (active) store_bf16x8(dO_c + (row * H + h) * D + j * 8, dxg);
+        } else if (threadIdx.x == 0) {
+            dgate_p[bt] = 0.0f;
         }
     }
-    // dp_t = z_t * sum_{h,d} dO (o~G - o~L)
-    dp_acc = head_sum(dp_acc, 32);
-    if ((threadIdx.x & 31) == 0) sh_dp[threadIdx.x >> 5] = dp_acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        float s = 0.f;
+    if (DGAIN) {
+        const int64_t hd = static_cast<int64_t>(nvec) * 8;
+        float* pl = part + static_cast<int64_t>(blockIdx.x) * 2 * hd;
 #pragma unroll
-        for (int w = 0; w < kThreads / 32; ++w) s += sh_dp[w];
-        dgate_p[bt] = sel ? s : 0.0f;
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            if (v < nvec) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    pl[v * 8 + i] = accL[k][i];
+                    pl[hd + v * 8 + i] = accG[k][i];
+                }
+            }
+        }
+    }
+}
+
+// dgain_{l,g}[e] = sum over blocks b (in order) of part[b][{0,1}][e].
+__global__ void __launch_bounds__(256) combine_dgain_reduce_kernel(const float* __restrict__ part, int nblk, int hd,
+                                                                   float* __restrict__ dgain_l,
+                                                                   float* __restrict__ dgain_g)
+{
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= 2 * hd) return;
+    const int w = e / hd, x = e % hd;
+    float s = 0.f;
+    for (int b = 0; b < nblk; ++b) s += part[(static_cast<int64_t>(b) * 2 + w) * hd + x];
+    float* dst = w == 0 ? dgain_l : dgain_g;
+    if (dst) dst[x] = s;
+}
+
+int vec_per_thread(const logo_dims& d)
+{
+    const int nvec = d.Hq * (d.D / 8);
+    const int need = (nvec + kThreads - 1) / kThreads;
+    return need <= 1 ? 1 : need <= 2 ? 2 : need <= 4 ? 4 : 8;
+}
+
+// One wave of resident blocks (the grid-stride loop gives every block the
+// same number of tokens), capped by the token count.
+template <typename K>
+int64_t wave_blocks(K kernel, int64_t ntok)
+{
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, 0) != cudaSuccess || per_sm < 1)
+        per_sm = 1;
+    const int64_t cap = static_cast<int64_t>(device_sm_count()) * per_sm;
+    return ntok < cap ? ntok : cap;
+}
+
+int64_t gains_blocks(const logo_dims& d)
+{
+    const int64_t ntok = static_cast<int64_t>(d.B) * d.T;
+    switch (vec_per_thread(d)) {
+        case 1: return wave_blocks(combine_bwd_kernel<1, true>, ntok);
+        case 2: return wave_blocks(combine_bwd_kernel<2, true>, ntok);
+        default: return wave_blocks(combine_bwd_kernel<4, true>, ntok);
     }
 }
 
@@ -193,6 +305,7 @@ int check_combine(const logo_dims& d)
     if (d.B < 1 || d.T < 1 || d.Hq < 1) return LOGO_ERR_INVALID_ARG;
     if (d.D != 64 && d.D != 128) return LOGO_ERR_UNSUPPORTED;
     if (static_cast<int64_t>(d.B) * d.T > (1ll << 30)) return LOGO_ERR_UNSUPPORTED;
+    if (d.Hq * (d.D / 8) > kMaxVec) return LOGO_ERR_UNSUPPORTED;  // Hq * D <= 16384
     return LOGO_OK;
 }
 
@@ -216,15 +329,25 @@ extern "C" int logo_combine(const logo_bf16* o_l, const logo_bf16* o_c, const fl
         (gain_g && !aligned16(gain_g)))
         return LOGO_ERR_UNSUPPORTED;
     const int64_t ntok = static_cast<int64_t>(dims.B) * dims.T;
-    combine_fwd_kernel<<<static_cast<unsigned>(ntok), kThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-        o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, o, rstd_l, rstd_g, dims.Hq, dims.D);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+#define LOGO_COMBINE_FWD(V)                                                                                       \
+    combine_fwd_kernel<V><<<static_cast<unsigned>(wave_blocks(combine_fwd_kernel<V>, ntok)), kThreads, 0, st>>>( \
+        o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, o, rstd_l, rstd_g, ntok, dims.Hq, dims.D)
+    switch (vec_per_thread(dims)) {
+        case 1: LOGO_COMBINE_FWD(1); break;
+        case 2: LOGO_COMBINE_FWD(2); break;
+        case 4: LOGO_COMBINE_FWD(4); break;
+        default: LOGO_COMBINE_FWD(8); break;
+    }
+#undef LOGO_COMBINE_FWD
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
-extern "C" int logo_combine_bwd(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p,
-                                const uint8_t* z, const int32_t* row_of, const float* gain_l, const float* gain_g,
-                                float eps, logo_bf16* dO_l, logo_bf16* dO_c, float* dgate_p, logo_dims dims,
-                                void* stream)
+namespace {
+int combine_bwd_common(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p,
+                       const uint8_t* z, const int32_t* row_of, const float* gain_l, const float* gain_g, float eps,
+                       logo_bf16* dO_l, logo_bf16* dO_c, float* dgate_p, float* dgain_l, float* dgain_g,
+                       void* workspace, size_t workspace_bytes, logo_dims dims, void* stream)
 {
     int rc = check_combine(dims);
     if (rc != LOGO_OK) return rc;
@@ -233,8 +356,70 @@ extern "C" int logo_combine_bwd(const logo_bf16* dO, const logo_bf16* o_l, const
     if (!aligned16(dO) || !aligned16(o_l) || !aligned16(o_c) || !aligned16(dO_l) || !aligned16(dO_c) ||
         (gain_l && !aligned16(gain_l)) || (gain_g && !aligned16(gain_g)))
         return LOGO_ERR_UNSUPPORTED;
+    const bool gains = dgain_l || dgain_g;
+    const int vpt = vec_per_thread(dims);
+    if (gains) {
+        if (dims.Hq * (dims.D / 8) > kMaxVecGains) return LOGO_ERR_UNSUPPORTED;  // Hq * D <= 8192
+        if (!workspace) return LOGO_ERR_INVALID_ARG;
+        if (workspace_bytes < logo_combine_bwd_workspace_size(dims)) return LOGO_ERR_WORKSPACE;
+    }
     const int64_t ntok = static_cast<int64_t>(dims.B) * dims.T;
-    combine_bwd_kernel<<<static_cast<unsigned>(ntok), kThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-        dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, dO_c, dgate_p, dims.Hq, dims.D);
-    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+    unsigned grid = 0;
+    float* part = static_cast<float*>(workspace);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+#define LOGO_COMBINE_BWD(V, G)                                                                                  \
+    grid = static_cast<unsigned>(wave_blocks(combine_bwd_kernel<V, G>, ntok));                                   \
+    combine_bwd_kernel<V, G><<<grid, kThreads, 0, st>>>(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, \
+                                                        dO_c, dgate_p, part, ntok, dims.Hq, dims.D)
+    if (gains) {
+        switch (vpt) {
+            case 1: LOGO_COMBINE_BWD(1, true); break;
+            case 2: LOGO_COMBINE_BWD(2, true); break;
+            default: LOGO_COMBINE_BWD(4, true); break;
+        }
+    } else {
+        switch (vpt) {
+            case 1: LOGO_COMBINE_BWD(1, false); break;
+            case 2: LOGO_COMBINE_BWD(2, false); break;
+            case 4: LOGO_COMBINE_BWD(4, false); break;
+            default: LOGO_COMBINE_BWD(8, false); break;
+        }
+    }
+#undef LOGO_COMBINE_BWD
+    if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    if (gains) {
+        const int hd = dims.Hq * dims.D;
+        combine_dgain_reduce_kernel<<<(2 * hd + 255) / 256, 256, 0, st>>>(part, static_cast<int>(grid), hd, dgain_l,
+                                                                          dgain_g);
+        if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    }
+    return LOGO_OK;
+}
+}  // namespace
+
+extern "C" int logo_combine_bwd(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c, const float* gate_p,
+                                const uint8_t* z, const int32_t* row_of, const float* gain_l, const float* gain_g,
+                                float eps, logo_bf16* dO_l, logo_bf16* dO_c, float* dgate_p, logo_dims dims,
+                                void* stream)
+{
+    return combine_bwd_common(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, dO_c, dgate_p, nullptr,
+                              nullptr, nullptr, 0, dims, stream);
+}
+
+extern "C" size_t logo_combine_bwd_workspace_size(logo_dims dims)
+{
+    if (check_combine(dims) != LOGO_OK) return 0;
+    if (dims.Hq * (dims.D / 8) > kMaxVecGains) return 0;
+    return static_cast<size_t>(gains_blocks(dims)) * 2 * static_cast<size_t>(dims.Hq) * dims.D * sizeof(float);
+}
+
+extern "C" int logo_combine_bwd_gains(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf16* o_c,
+                                      const float* gate_p, const uint8_t* z, const int32_t* row_of,
+                                      const float* gain_l, const float* gain_g, float eps, logo_bf16* dO_l,
+                                      logo_bf16* dO_c, float* dgate_p, float* dgain_l, float* dgain_g,
+                                      logo_dims dims, void* workspace, size_t workspace_bytes, void* stream)
+{
+    if (!dgain_l && !dgain_g) return LOGO_ERR_INVALID_ARG;
+    return combine_bwd_common(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, dO_c, dgate_p, dgain_l,
+                              dgain_g, workspace, workspace_bytes, dims, stream);
 }

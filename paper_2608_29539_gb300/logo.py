@@ -77,6 +77,9 @@ _SIGS = {
                                              _c_float, _vp, _c_size, _vp]),
     "logo_combine": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_float, _vp, _vp, _vp, Dims, _vp]),
     "logo_combine_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_float, _vp, _vp, _vp, Dims, _vp]),
+    "logo_combine_bwd_workspace_size": (_c_size, [Dims]),
+    "logo_combine_bwd_gains": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_float, _vp, _vp, _vp, _vp, _vp,
+                                        Dims, _vp, _c_size, _vp]),
 }
 
 
@@ -142,7 +145,8 @@ def _workspace(nbytes: int, device, ws=None):
 def workspace_bytes(kind: str, dims: Dims) -> int:
     fn = {"select": "logo_select_workspace_size", "local_bwd": "logo_local_attn_bwd_workspace_size",
           "global_fwd": "logo_global_attn_fwd_workspace_size",
-          "global_bwd": "logo_global_attn_bwd_workspace_size"}[kind]
+          "global_bwd": "logo_global_attn_bwd_workspace_size",
+          "combine_bwd_gains": "logo_combine_bwd_workspace_size"}[kind]
     return int(getattr(lib(), fn)(dims))
 
 
@@ -367,3 +371,25 @@ def logo_combine_bwd(dO, o_l, o_c, gate_p, z, row_of, gain_l=None, gain_g=None, 
     _call("logo_combine_bwd", _p(dO), _p(o_l), _p(o_c), _p(gate_p), _p(z), _p(row_of), _p(gain_l), _p(gain_g),
           float(eps), _p(dO_l), _p(dO_c), _p(dgate_p), d, _stream())
     return dO_l, dO_c, dgate_p
+
+
+def logo_combine_bwd_gains(dO, o_l, o_c, gate_p, z, row_of, gain_l=None, gain_g=None, eps: float = 1e-6,
+                           dO_l=None, dO_c=None, dgate_p=None, dgain_l=None, dgain_g=None, workspace=None):
+    """logo_combine_bwd plus the ContextNorm gain gradients (Eq. 9).
+    Returns (dO_l, dO_c, dgate_p, dgain_l, dgain_g); the gain gradients are
+    [Hq, D] float32."""
+    _need(dO, torch.bfloat16, "dO")
+    B, T, H, D = o_l.shape
+    d = Dims(B, T, H, H, D)
+    dev = o_l.device
+    dO_l = dO_l if dO_l is not None else torch.empty_like(o_l)
+    dO_c = dO_c if dO_c is not None else torch.empty((B * T, H, D), dtype=torch.bfloat16, device=dev)
+    dgate_p = dgate_p if dgate_p is not None else torch.empty((B, T), dtype=torch.float32, device=dev)
+    dgain_l = dgain_l if dgain_l is not None else torch.empty((H, D), dtype=torch.float32, device=dev)
+    dgain_g = dgain_g if dgain_g is not None else torch.empty((H, D), dtype=torch.float32, device=dev)
+    nbytes = int(lib().logo_combine_bwd_workspace_size(d))
+    ws = _workspace(nbytes, dev, workspace)
+    _call("logo_combine_bwd_gains", _p(dO), _p(o_l), _p(o_c), _p(gate_p), _p(z), _p(row_of), _p(gain_l),
+          _p(gain_g), float(eps), _p(dO_l), _p(dO_c), _p(dgate_p), _p(dgain_l), _p(dgain_g), d, _p(ws),
+          ws.numel(), _stream())
+    return dO_l, dO_c, dgate_p, dgain_l, dgain_g

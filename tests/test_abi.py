@@ -125,6 +125,30 @@ def test_decode_host_checks(lib):
                                             null) == logo.LOGO_ERR_UNSUPPORTED
 
 
+def test_combine_gains_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    d = logo.Dims(2, 300, 4, 4, 128)
+    null = None
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected before use
+    f = ctypes.c_float
+    ws = L.logo_combine_bwd_workspace_size(d)
+    assert ws >= 2 * 4 * 128 * 4  # at least one block's two [H, D] partial sums
+    assert L.logo_combine_bwd_workspace_size(logo.Dims(2, 300, 72, 72, 128)) == 0  # Hq*D > 8192
+    args = lambda dgl, dgg, dims, w, wb: (fake, fake, fake, fake, fake, fake, null, null, f(1e-6), fake, fake,  # noqa: E731
+                                          fake, dgl, dgg, dims, w, wb, null)
+    assert L.logo_combine_bwd_gains(*args(null, null, d, fake, ws)) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_combine_bwd_gains(*args(fake, fake, d, null, ws)) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_combine_bwd_gains(*args(fake, fake, d, fake, 16)) == logo.LOGO_ERR_WORKSPACE
+    assert L.logo_combine_bwd_gains(*args(fake, null, logo.Dims(2, 300, 72, 72, 128), fake,
+                                          1 << 30)) == logo.LOGO_ERR_UNSUPPORTED
+    assert L.logo_combine_bwd_gains(*args(fake, fake, logo.Dims(2, 300, 4, 4, 96), fake,
+                                          ws)) == logo.LOGO_ERR_UNSUPPORTED
+    # the plain combine calls reject Hq*D > 16384
+    assert L.logo_combine(fake, fake, fake, fake, fake, null, null, f(1e-6), fake, null, null,
+                          logo.Dims(1, 8, 130, 130, 128), null) == logo.LOGO_ERR_UNSUPPORTED
+
+
 def test_workspace_sizes_grow_with_shape(lib):
     from paper_2608_29539_gb300 import logo
     L = logo.lib()

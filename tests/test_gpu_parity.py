@@ -269,6 +269,35 @@ def test_combine_bwd(B, T, H, D, ratio, gains):
     assert (np32(dp)[zn == 0] == 0).all()
 
 
+GAIN_CASES = COMBINE_CASES + [
+    (1, 700, 64, 128, 0.125, True),  # Hq*D = 8192, the largest supported: four vectors per thread
+    (3, 77, 1, 64, 0.3, False),      # one head: most threads of a block idle
+]
+
+
+@pytest.mark.parametrize("B,T,H,D,ratio,gains", GAIN_CASES)
+def test_combine_bwd_gains(B, T, H, D, ratio, gains):
+    p, (z, row_of), n, o_l, o_c, gl, gg = _combine_setup(B, T, H, D, ratio, gains, seed=3 * T + H)
+    dO = seeded((B, T, H, D), 7 * T, torch.bfloat16)
+    cu = lambda t: None if t is None else t.cuda()  # noqa: E731
+    args = (dO.cuda(), o_l.cuda(), o_c.cuda(), p.cuda(), z, row_of, cu(gl), cu(gg), 1e-6)
+    plain = L().logo_combine_bwd(*args)
+    with_gains = L().logo_combine_bwd_gains(*args)
+    again = L().logo_combine_bwd_gains(*args)
+    torch.cuda.synchronize()
+    # the same input gradients as the plain call, bit for bit
+    assert torch.equal(plain[0], with_gains[0]) and torch.equal(plain[2], with_gains[2])
+    assert torch.equal(plain[1][:n], with_gains[1][:n])
+    # deterministic: blocks are summed in a fixed order
+    assert torch.equal(with_gains[3], again[3]) and torch.equal(with_gains[4], again[4])
+    zn, rown = z.cpu().numpy(), row_of.cpu().numpy()
+    rgl, rgg = oracle.combine_dgain(np32(dO), np32(o_l), np32(o_c)[:n], np32(p), zn, rown, 1e-6)
+    check_close(np32(with_gains[3]), rgl, "dgain_l")
+    check_close(np32(with_gains[4]), rgg, "dgain_g")
+    if n == 0:
+        assert bool((with_gains[4] == 0).all())
+
+
 # --------------------------------------------------- whole step, small workload
 def test_layer_step_4k_workload():
     """The 4K workload end to end through the layer chain; every call checked
