@@ -82,6 +82,8 @@ def _load():
                                                _f64p, _f64p, _f64p]
             lib.oracle_combine_dgain.argtypes = [_f32p, _f32p, _f32p, _f32p, _u8p, _i32p, ctypes.c_double,
                                                  _int, _int, _int, _int, _f64p, _f64p]
+            lib.oracle_gate.argtypes = [_f32p, _f32p, _i64, _int, _f64p]
+            lib.oracle_gate_bwd.argtypes = [_f32p, _f32p, _f32p, _i64, _int, _f64p, _f64p]
             lib.oracle_num_threads.restype = _int
             _lib = lib
     return _lib
@@ -274,3 +276,27 @@ def combine_dgain(dO, oL, oGc, p, z, row_of, eps: float = 1e-6):
     _load().oracle_combine_dgain(_f32(dO), oL, oGc, _f32(p), np.ascontiguousarray(z, dtype=np.uint8),
                                  _i32(row_of), float(eps), B, T, H, D, dgL, dgG)
     return dgL, dgG
+
+
+def gate(x, w):
+    """Eq. 7: p = sigmoid(x . w_g) per token.  x [..., dm], w [dm]; returns p
+    [...] float64."""
+    x = _f32(x)
+    dm = x.shape[-1]
+    n = x.size // dm if dm else 0
+    p = np.zeros(n, dtype=np.float64)
+    if n:
+        _load().oracle_gate(x.reshape(n, dm), _f32(w).reshape(dm), n, dm, p)
+    return p.reshape(x.shape[:-1])
+
+
+def gate_bwd(x, w, dp):
+    """Backward of gate for the given dp: (dx [..., dm], dw [dm]) float64."""
+    x = _f32(x)
+    dm = x.shape[-1]
+    n = x.size // dm
+    dx = np.zeros((n, dm), dtype=np.float64)
+    dw = np.zeros(dm, dtype=np.float64)
+    if n:
+        _load().oracle_gate_bwd(x.reshape(n, dm), _f32(w).reshape(dm), _f32(dp).reshape(n), n, dm, dx, dw)
+    return dx.reshape(x.shape), dw

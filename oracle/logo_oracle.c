@@ -37,6 +37,35 @@ void oracle_select_threshold(const float* p, int64_t n, float b_th, uint8_t* z)
     for (int64_t i = 0; i < n; ++i) z[i] = (p[i] > b_th) ? 1 : 0;
 }
 
+/* Eq. 7 gate: p_t = sigmoid(x_t . w_g) in double, x [N, dm] (float32 holding
+ * the bf16 values the GPU reads), w_g [dm]. */
+void oracle_gate(const float* x, const float* w, int64_t n, int dm, double* p)
+{
+    for (int64_t t = 0; t < n; ++t) {
+        double a = 0.0;
+        for (int i = 0; i < dm; ++i) a += (double)x[t * dm + i] * (double)w[i];
+        p[t] = 1.0 / (1.0 + exp(-a));
+    }
+}
+
+/* Backward of oracle_gate for a given dp: with p recomputed in double,
+ * dlogit_t = dp_t p_t (1 - p_t) (the sigmoid's derivative),
+ * dx_t = dlogit_t w_g, dw_g = sum over t (in order) of dlogit_t x_t. */
+void oracle_gate_bwd(const float* x, const float* w, const float* dp, int64_t n, int dm, double* dx, double* dw)
+{
+    memset(dw, 0, sizeof(double) * (size_t)dm);
+    for (int64_t t = 0; t < n; ++t) {
+        double a = 0.0;
+        for (int i = 0; i < dm; ++i) a += (double)x[t * dm + i] * (double)w[i];
+        double pt = 1.0 / (1.0 + exp(-a));
+        double g = (double)dp[t] * pt * (1.0 - pt);
+        for (int i = 0; i < dm; ++i) {
+            dx[t * dm + i] = g * (double)w[i];
+            dw[i] += g * (double)x[t * dm + i];
+        }
+    }
+}
+
 /* Eq. 3 and Eq. 11 (Sec. 3.2, Budget Control): the realised ratio is
  * F = n_sel / n_valid, and the threshold moves by gamma * sign(F - rho).
  * F and the sign are evaluated in double from the integer counts; b_th and

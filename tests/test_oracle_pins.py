@@ -482,6 +482,49 @@ def test_gain_grads_finite_differences_and_special_cases():
     np.testing.assert_allclose(dgL0, ref, rtol=1e-12, atol=1e-12)
 
 
+def test_gate_matches_numpy_and_closed_forms():
+    rng = np.random.default_rng(11)
+    x = rng.standard_normal((3, 17, 64)).astype(np.float32)
+    w = (0.1 * rng.standard_normal(64)).astype(np.float32)
+    p = oracle.gate(x, w)
+    logit = x.astype(np.float64) @ w.astype(np.float64)
+    np.testing.assert_allclose(p, 1.0 / (1.0 + np.exp(-logit)), rtol=1e-14)
+    np.testing.assert_allclose(p, torch.sigmoid(torch.tensor(logit)).numpy(), rtol=1e-14)
+    # near-zero init of the gate (Sec. 3.2): w = 0 puts every p at exactly 0.5
+    assert (oracle.gate(x, np.zeros(64, np.float32)) == 0.5).all()
+    # one active coordinate: p = sigmoid(x_i w_i); opposite inputs give 1 - p
+    e = np.zeros(64, np.float32)
+    e[5] = 2.0
+    np.testing.assert_allclose(oracle.gate(x, e), 1 / (1 + np.exp(-2.0 * x[..., 5].astype(np.float64))), rtol=1e-14)
+    np.testing.assert_allclose(oracle.gate(-x, w), 1.0 - p, rtol=1e-12, atol=1e-15)
+
+
+def test_gate_bwd_matches_torch_autograd_and_finite_differences():
+    rng = np.random.default_rng(12)
+    x = rng.standard_normal((2, 9, 32)).astype(np.float32)
+    w = (0.2 * rng.standard_normal(32)).astype(np.float32)
+    dp = rng.standard_normal((2, 9)).astype(np.float32)
+    dx, dw = oracle.gate_bwd(x, w, dp)
+    tx = torch.tensor(x, dtype=torch.float64, requires_grad=True)
+    tw = torch.tensor(w, dtype=torch.float64, requires_grad=True)
+    torch.sigmoid(tx @ tw).backward(torch.tensor(dp, dtype=torch.float64))
+    np.testing.assert_allclose(dx, tx.grad.numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(dw, tw.grad.numpy(), rtol=1e-12, atol=1e-15)
+    loss = lambda w_: float((oracle.gate(x, w_) * dp.astype(np.float64)).sum())  # noqa: E731
+    for i in (0, 13, 31):
+        hi, lo = w.copy(), w.copy()
+        hi[i] += np.float32(1e-3)
+        lo[i] -= np.float32(1e-3)
+        fd = (loss(hi) - loss(lo)) / (float(hi[i]) - float(lo[i]))
+        assert fd == pytest.approx(dw[i], rel=1e-5, abs=1e-9)
+    # dp = 0 passes no gradient; w = 0 gives dlogit = dp / 4 and dx = 0
+    dx0, dw0 = oracle.gate_bwd(x, w, np.zeros_like(dp))
+    assert (dx0 == 0).all() and (dw0 == 0).all()
+    dxz, dwz = oracle.gate_bwd(x, np.zeros_like(w), dp)
+    assert (dxz == 0).all()
+    np.testing.assert_allclose(dwz, (dp.astype(np.float64)[..., None] / 4 * x).sum(axis=(0, 1)), rtol=1e-12)
+
+
 def test_ratio_zero_layer_is_pure_local():
     # rho = 0: no token is selected, the layer output is Norm^L(O^L) and no
     # gradient reaches the global branch or the gate.
