@@ -11,6 +11,10 @@
  *   logo_global_sparse_attn_fwd / _bwd
  *                                Eq. 8 global branch on the selected rows only
  *   logo_combine / _bwd          Eq. 9 ContextNorm + Eq. 10 gate-weighted fusion
+ *   logo_combine_bwd_gains       ... plus the gradients of the ContextNorm gains
+ *   logo_gate_select / logo_gate_bwd
+ *                                Eq. 7 gate p = sigmoid(x . w_g) fused ahead of
+ *                                logo_select, and its backward
  *
  * Conventions shared by every entry point
  *   - All tensor pointers are DEVICE pointers owned by the caller.  The
@@ -260,6 +264,39 @@ LOGO_API int logo_global_sparse_attn_bwd(const logo_bf16* q, const logo_bf16* k,
                                 const float* lse_c, const logo_bf16* dO_c, logo_bf16* dq, logo_bf16* dk,
                                 logo_bf16* dv, logo_dims dims, float scale, void* workspace,
                                 size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * logo_gate_select -- the token gate of Eq. 7, p_t = sigmoid(x_t . w_g), then
+ *   logo_select on p: the gate and the selection in one call.
+ * In : x [B,T,d_model] bf16 (the layer input; rows contiguous, 16-byte
+ *      aligned); w_g [d_model] float32 (16-byte aligned); d_model a multiple
+ *      of 8 and at most 8192; mode / b_th / ratio as logo_select.  Only dims.B
+ *      and dims.T are read.
+ * Out: gate_p [B,T] float32: the p the selection compared (fp32 dot product
+ *      over d_model, fp32 sigmoid); z, pos, cu_q, row_of, n_sel_total as
+ *      logo_select.
+ * Workspace: logo_select_workspace_size(dims) bytes.
+ * Errors: as logo_select; LOGO_ERR_UNSUPPORTED for d_model or alignment. */
+LOGO_API int logo_gate_select(const logo_bf16* x, const float* w_g, int d_model, logo_dims dims, int mode,
+                              float b_th, float ratio, float* gate_p, uint8_t* z, int32_t* pos, int32_t* cu_q,
+                              int32_t* row_of, int32_t* n_sel_total, void* workspace, size_t workspace_bytes,
+                              void* stream);
+
+/* logo_gate_bwd -- backward of the gate with the selection held fixed (z
+ *   passes no gradient): dlogit_t = dp_t p_t (1 - p_t), dx_t = dlogit_t w_g,
+ *   dw_g = sum over t of dlogit_t x_t.
+ * In : x, w_g, d_model as logo_gate_select; gate_p [B,T] float32 (its
+ *      output); dgate_p [B,T] float32 (e.g. from logo_combine_bwd).
+ * Out: dx [B,T,d_model] bf16: written, or added to when accumulate = 1 (the
+ *      caller's gradient of x from its other uses); may be NULL.  dw_g
+ *      [d_model] float32, overwritten; may be NULL (not both).  dw_g is summed
+ *      per block, then over the blocks in a fixed order (deterministic).
+ * Workspace: logo_gate_bwd_workspace_size(dims, d_model) bytes when dw_g is
+ *      requested (else may be NULL). */
+LOGO_API size_t logo_gate_bwd_workspace_size(logo_dims dims, int d_model);
+LOGO_API int logo_gate_bwd(const logo_bf16* x, const float* w_g, const float* gate_p, const float* dgate_p,
+                           int d_model, logo_dims dims, logo_bf16* dx, int accumulate, float* dw_g, void* workspace,
+                           size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * logo_combine -- ContextNorm per branch (Eq. 9: head-wise RMSNorm over D,

@@ -57,6 +57,10 @@ _SIGS = {
     "logo_num_sms": (_c_int, []),
     "logo_select_workspace_size": (_c_size, [Dims]),
     "logo_select": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
+    "logo_gate_select": (_c_int, [_vp, _vp, _c_int, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp,
+                                  _vp, _c_size, _vp]),
+    "logo_gate_bwd_workspace_size": (_c_size, [Dims, _c_int]),
+    "logo_gate_bwd": (_c_int, [_vp, _vp, _vp, _vp, _c_int, Dims, _vp, _c_int, _vp, _vp, _c_size, _vp]),
     "logo_select_noalloc": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp]),
     "logo_select_device_threshold": (_c_int, [_vp, Dims, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
     "logo_budget_update": (_c_int, [_vp, Dims, _c_float, _c_float, _vp, _vp, _vp]),
@@ -178,6 +182,52 @@ def logo_select(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None
     _call("logo_select", _p(gate_p), dims, int(mode), float(b_th), float(ratio), _p(z), _p(pos), _p(cu_q),
           _p(row_of), _p(n_sel_total), _p(ws), nbytes, _stream())
     return z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_gate_select(x, w_g, mode: int, b_th: float = 0.5, ratio: float = 0.0, gate_p=None, z=None, pos=None,
+                     cu_q=None, row_of=None, n_sel_total=None, workspace=None):
+    """Eq. 7 gate p = sigmoid(x . w_g) (x [B, T, d_model] bf16, w_g [d_model]
+    float32) followed by the routing of logo_select.  Returns
+    (gate_p, z, pos, cu_q, row_of, n_sel_total)."""
+    _need(x, torch.bfloat16, "x")
+    _need(w_g, torch.float32, "w_g")
+    B, T, dm = x.shape
+    dev = x.device
+    dims = Dims(B, T, 1, 1, 64)
+    gate_p = gate_p if gate_p is not None else torch.empty((B, T), dtype=torch.float32, device=dev)
+    z = z if z is not None else torch.empty((B, T), dtype=torch.uint8, device=dev)
+    pos = pos if pos is not None else torch.empty((B * T,), dtype=torch.int32, device=dev)
+    cu_q = cu_q if cu_q is not None else torch.empty((B + 1,), dtype=torch.int32, device=dev)
+    row_of = row_of if row_of is not None else torch.empty((B, T), dtype=torch.int32, device=dev)
+    n_sel_total = n_sel_total if n_sel_total is not None else torch.empty((1,), dtype=torch.int32, device=dev)
+    nbytes = workspace_bytes("select", dims)
+    ws = _workspace(nbytes, dev, workspace)
+    _call("logo_gate_select", _p(x), _p(w_g), int(dm), dims, int(mode), float(b_th), float(ratio), _p(gate_p), _p(z),
+          _p(pos), _p(cu_q), _p(row_of), _p(n_sel_total), _p(ws), nbytes, _stream())
+    return gate_p, z, pos, cu_q, row_of, n_sel_total
+
+
+def logo_gate_bwd(x, w_g, gate_p, dgate_p, dx=None, accumulate: bool = False, dw_g=None, want_dx: bool = True,
+                  want_dw: bool = True, workspace=None):
+    """Backward of the gate: dx = dlogit w_g (written, or added to dx when
+    accumulate), dw_g = sum_t dlogit_t x_t with dlogit = dp p (1 - p).
+    Returns (dx, dw_g) (None for a part not asked for)."""
+    _need(x, torch.bfloat16, "x")
+    B, T, dm = x.shape
+    dev = x.device
+    dims = Dims(B, T, 1, 1, 64)
+    if want_dx and dx is None:
+        if accumulate:
+            raise ValueError("accumulate needs the dx to add to")
+        dx = torch.empty_like(x)
+    if not want_dx:
+        dx = None
+    dw_g = (dw_g if dw_g is not None else torch.empty((dm,), dtype=torch.float32, device=dev)) if want_dw else None
+    nbytes = int(lib().logo_gate_bwd_workspace_size(dims, dm)) if want_dw else 0
+    ws = _workspace(nbytes, dev, workspace) if want_dw else None
+    _call("logo_gate_bwd", _p(x), _p(w_g), _p(gate_p), _p(dgate_p), int(dm), dims, _p(dx), int(bool(accumulate)),
+          _p(dw_g), _p(ws), nbytes, _stream())
+    return dx, dw_g
 
 
 def logo_select_device_threshold(gate_p, b_th, z=None, pos=None, cu_q=None, row_of=None, n_sel_total=None,

@@ -149,6 +149,35 @@ def test_combine_gains_host_checks(lib):
                           logo.Dims(1, 8, 130, 130, 128), null) == logo.LOGO_ERR_UNSUPPORTED
 
 
+def test_gate_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    d = logo.Dims(2, 300, 1, 1, 64)
+    null = None
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected before use
+    odd = ctypes.c_void_p((1 << 20) + 2)
+    f = ctypes.c_float
+    ws = L.logo_select_workspace_size(d)
+    sel = lambda x, w, dm, mode, ratio, wsz: L.logo_gate_select(x, w, dm, d, mode, f(0.5), f(ratio), fake, fake,  # noqa: E731
+                                                                  fake, fake, fake, fake, fake, wsz, null)
+    assert sel(fake, fake, 4096, 1, 0.125, ws - 1) == logo.LOGO_ERR_WORKSPACE
+    for dm in (0, 4, 100, 8200):
+        assert sel(fake, fake, dm, 1, 0.125, ws) == logo.LOGO_ERR_UNSUPPORTED
+    assert sel(null, fake, 4096, 1, 0.125, ws) == logo.LOGO_ERR_INVALID_ARG
+    assert sel(fake, fake, 4096, 3, 0.125, ws) == logo.LOGO_ERR_INVALID_ARG
+    assert sel(fake, fake, 4096, 1, 1.5, ws) == logo.LOGO_ERR_INVALID_ARG
+    assert sel(odd, fake, 4096, 1, 0.125, ws) == logo.LOGO_ERR_UNSUPPORTED
+    wb = L.logo_gate_bwd_workspace_size(d, 4096)
+    assert wb >= 4096 * 4 and L.logo_gate_bwd_workspace_size(d, 8200) == 0
+    bwd = lambda dx, acc, dw, w, wsz: L.logo_gate_bwd(fake, fake, fake, fake, 4096, d, dx, acc, dw, w, wsz,  # noqa: E731
+                                                     null)
+    assert bwd(null, 0, null, fake, wb) == logo.LOGO_ERR_INVALID_ARG
+    assert bwd(fake, 2, fake, fake, wb) == logo.LOGO_ERR_INVALID_ARG
+    assert bwd(fake, 0, fake, null, wb) == logo.LOGO_ERR_WORKSPACE
+    assert bwd(fake, 0, fake, fake, wb - 4) == logo.LOGO_ERR_WORKSPACE
+    assert bwd(odd, 0, null, null, 0) == logo.LOGO_ERR_UNSUPPORTED
+
+
 def test_workspace_sizes_grow_with_shape(lib):
     from paper_2608_29539_gb300 import logo
     L = logo.lib()
