@@ -63,6 +63,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-routing", action="store_true")
+    ap.add_argument("--no-fusions", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     return ap.parse_args()
 
@@ -356,6 +357,67 @@ def routing_bench(layer, x, w, dev):
             "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
 
 
+def fusions_bench(layer, x, w, dev, pk):
+    """The fused pieces around the attention: the Eq. 7 gate + select on a
+    [B, T, d_model = Hq*D] input, the gate backward (dx accumulated into the
+    caller's gradient, dw_g), and the combine backward with the ContextNorm
+    gain gradients against the one without.  Bytes are the HBM bytes each call
+    must move at least; every operand is at least 128 MiB (about L2's size)."""
+    from paper_2608_29539_gb300 import logo as L
+    dm = w.Hq * w.D
+    g = torch.Generator(device=dev).manual_seed(5)
+    xin = torch.randn((w.B, w.T, dm), generator=g, device=dev).to(torch.bfloat16)
+    wg = torch.randn((dm,), generator=g, device=dev) / dm ** 0.5
+    dxin = torch.randn((w.B, w.T, dm), generator=g, device=dev).to(torch.bfloat16)
+    bufs = (torch.empty((w.B, w.T), dtype=torch.float32, device=dev), torch.empty_like(layer.z),
+            torch.empty_like(layer.pos), torch.empty_like(layer.cu_q), torch.empty_like(layer.row_of),
+            torch.empty_like(layer.n_sel))
+    c = layer.cfg
+    dw = torch.empty((dm,), dtype=torch.float32, device=dev)
+    gws = torch.empty((int(L.lib().logo_gate_bwd_workspace_size(L.Dims(w.B, w.T, 1, 1, 64), dm)),), dtype=torch.uint8,
+                      device=dev)
+    cws = torch.empty((L.workspace_bytes("combine_bwd_gains", layer.dims),), dtype=torch.uint8, device=dev)
+    dgl = torch.empty((w.Hq, w.D), dtype=torch.float32, device=dev)
+    dgg = torch.empty_like(dgl)
+    n = int(layer.n_sel[0])
+
+    def timed(fn, reps=20):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    gate = lambda: L.logo_gate_select(xin, wg, c.mode, c.b_th, c.ratio, *bufs, workspace=layer.ws)  # noqa: E731
+    gate_bwd = lambda: L.logo_gate_bwd(xin, wg, bufs[0], layer.dgate, dx=dxin, accumulate=True, dw_g=dw,  # noqa: E731
+                                       workspace=gws)
+    cargs = (x["dO"], layer.o_l, layer.o_c, x["p"], layer.z, layer.row_of, None, None, c.eps, layer.dO_l, layer.dO_c,
+             layer.dgate)
+    cplain = lambda: L.logo_combine_bwd(*cargs)  # noqa: E731
+    cgains = lambda: L.logo_combine_bwd_gains(*cargs, dgain_l=dgl, dgain_g=dgg, workspace=cws)  # noqa: E731
+    tok_row = w.Hq * w.D * 2
+    ntok = w.B * w.T
+    out = {}
+    ms = timed(gate)
+    byts = ntok * dm * 2 + ntok * 4
+    out["gate_select"] = {"ms": ms, "GB_per_s": byts / ms / 1e6, "frac_of_hbm_peak": byts / ms / 1e6 / pk["hbm"],
+                          "bytes": byts, "d_model": dm, "launches": 5}
+    ms = timed(gate_bwd)
+    byts = 3 * ntok * dm * 2 + 2 * ntok * 4
+    out["gate_bwd"] = {"ms": ms, "GB_per_s": byts / ms / 1e6, "frac_of_hbm_peak": byts / ms / 1e6 / pk["hbm"],
+                       "bytes": byts, "note": "x read, dx read and written (accumulated), dw_g", "launches": 2}
+    ms_p, ms_g = timed(cplain), timed(cgains)
+    byts = 3 * ntok * tok_row + 2 * n * tok_row
+    out["combine_bwd_gains"] = {"ms": ms_g, "ms_without_gains": ms_p, "GB_per_s": byts / ms_g / 1e6,
+                                "frac_of_hbm_peak": byts / ms_g / 1e6 / pk["hbm"], "bytes": byts, "launches": 2}
+    return out
+
+
 def decode_bench(dev, pk):
     """Time one decoding step's attention (local branch from ring caches, global
     branch for the selected sequences only, fusion) and the same step under the
@@ -513,6 +575,11 @@ def native_arm(a, rank, world, local_rank, dist_on):
     # threshold on the device, then the Eq. 11 update, on this workload's gates
     if not a.no_routing:
         line["device_routing_loop"] = routing_bench(layer, x, w, dev)
+
+    # ---- the fused gate (Eq. 7) + select, its backward, and the combine
+    # backward with the ContextNorm gain gradients
+    if not a.no_fusions:
+        line["fusions"] = fusions_bench(layer, x, w, dev, pk)
 
     # ---- one decoding step (Sec. 3.3): 32 sequences with 16K-token caches,
     # GQA 32/8, d = 128, W = 1024, about 1/8 of the new tokens selected

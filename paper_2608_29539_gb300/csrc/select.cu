@@ -68,14 +68,88 @@ __device__ __forceinline__ int block_excl_scan(int v, int* total, int* sh_warp)
     return base + x - v;
 }
 
+// Radix histograms for 1024-thread blocks: each warp counts into its own
+// copy (contention stays inside a warp however the keys cluster), then the
+// copies are summed per bin.
+struct WarpHist {
+    int h[32][256];
+};
+
+__device__ __forceinline__ void hist_clear(WarpHist& wh)
+{
+    int* f = &wh.h[0][0];
+    for (int i = threadIdx.x; i < 32 * 256; i += blockDim.x) f[i] = 0;
+}
+
+__device__ __forceinline__ void hist_sum(const WarpHist& wh, int* hist)
+{
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+        int s = 0;
+#pragma unroll 8
+        for (int w = 0; w < 32; ++w) s += wh.h[w][i];
+        hist[i] = s;
+    }
+}
+
+// Count one key per lane into the warp's histogram (every lane of the warp
+// calls this together).  The top byte of a gate's key is its sign and
+// exponent, so in the first pass nearly every key of (0, 1) gates falls in one
+// or two bins: there, lanes with the same bin are grouped and one atomic adds
+// the group's size.  Later passes spread over many bins, and a plain atomic
+// per lane is cheaper than the grouping.
+__device__ __forceinline__ void count_key(WarpHist& wh, int warp, bool in, uint32_t key, int shift)
+{
+    const uint32_t bin = (key >> shift) & 0xFFu;
+    if (shift == 24) {
+        const unsigned same = __match_any_sync(0xffffffffu, in ? bin : 0x100u);
+        if (in && (threadIdx.x & 31) == __ffs(same) - 1) atomicAdd(&wh.h[warp][bin], __popc(same));
+    } else if (in) {
+        atomicAdd(&wh.h[warp][bin], 1);
+    }
+}
+
+// Warp 0: the bin holding the `remaining`-th largest key counted from the top,
+// and how many keys of that bin still have to be taken (bins scanned from 255
+// down, lane l holding bins 255-8l .. 248-8l).
+__device__ __forceinline__ void hist_pick(const int* hist, int remaining, uint32_t prefix, int shift,
+                                          uint32_t* sh_prefix, int* sh_remaining)
+{
+    const int lane = threadIdx.x & 31;
+    int c[8], sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        c[i] = hist[255 - 8 * lane - i];
+        sum += c[i];
+    }
+    int incl = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    const unsigned reach = __ballot_sync(0xffffffffu, incl >= remaining);
+    const int owner = reach ? __ffs(reach) - 1 : 31;
+    if (lane == owner) {
+        int above = incl - sum;
+        int d = 255 - 8 * lane;
+        for (int i = 0; i < 8; ++i, --d) {
+            if (above + c[i] >= remaining || d == 0) break;
+            above += c[i];
+        }
+        *sh_prefix = prefix | (static_cast<uint32_t>(d) << shift);
+        *sh_remaining = remaining - above;
+    }
+}
+
 // Ratio mode: find, per sequence, the key of the k-th largest gate.
 __global__ void __launch_bounds__(1024) radix_select_kernel(const float* __restrict__ p, int T, int k,
                                                             SeqThresh* __restrict__ out)
 {
+    __shared__ WarpHist wh;
     __shared__ int hist[256];
     __shared__ uint32_t sh_prefix;
     __shared__ int sh_remaining;
-    const int b = blockIdx.x;
+    const int b = blockIdx.x, warp = threadIdx.x >> 5;
     const float* pb = p + static_cast<int64_t>(b) * T;
     if (k <= 0) {
         if (threadIdx.x == 0) out[b] = SeqThresh{0xFFFFFFFFu, 0};
@@ -88,23 +162,25 @@ __global__ void __launch_bounds__(1024) radix_select_kernel(const float* __restr
     uint32_t prefix = 0, mask = 0;
     int remaining = k;
     for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+        hist_clear(wh);
         __syncthreads();
-        for (int t = threadIdx.x; t < T; t += blockDim.x) {
-            uint32_t key = gate_key(pb[t]);
-            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xFFu], 1);
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int above = 0;
-            int d = 255;
-            for (; d > 0; --d) {
-                if (above + hist[d] >= remaining) break;
-                above += hist[d];
+        // eight loads per thread in flight before the counting
+        for (int base = 0; base < T; base += 8 * blockDim.x) {
+            uint32_t keys[8];
+            bool valid[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int t = base + u * blockDim.x + threadIdx.x;
+                valid[u] = t < T;
+                keys[u] = valid[u] ? gate_key(pb[t]) : 0u;
             }
-            sh_prefix = prefix | (static_cast<uint32_t>(d) << shift);
-            sh_remaining = remaining - above;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) count_key(wh, warp, valid[u] && (keys[u] & mask) == prefix, keys[u], shift);
         }
+        __syncthreads();
+        hist_sum(wh, hist);
+        __syncthreads();
+        if (warp == 0) hist_pick(hist, remaining, prefix, shift, &sh_prefix, &sh_remaining);
         __syncthreads();
         prefix = sh_prefix;
         remaining = sh_remaining;
@@ -112,6 +188,155 @@ __global__ void __launch_bounds__(1024) radix_select_kernel(const float* __restr
         __syncthreads();
     }
     if (threadIdx.x == 0) out[b] = SeqThresh{prefix, remaining};
+}
+
+// Ratio mode, T <= 1024 * KPT: the whole selection of one sequence in one
+// block of 1024 threads.  Every sequence selects exactly k_eff tokens, so
+// sequence b's packed rows start at b * k_eff and no scan across sequences is
+// needed.  A thread owns KPT consecutive tokens (keys kept in registers for
+// the four radix passes), so block-wide scans in thread order are scans in t.
+// The gates come in, and z / row_of go out, through shared memory with
+// coalesced accesses (a thread's own tokens are KPT words apart from its
+// neighbours': read or written straight from global memory they cost one
+// sector per lane per access on the block's single SM).
+template <int KPT>
+__global__ void __launch_bounds__(1024) select_ratio_small_kernel(const float* __restrict__ p, int B, int T, int k,
+                                                                  uint8_t* __restrict__ z, int32_t* __restrict__ pos,
+                                                                  int32_t* __restrict__ cu_q,
+                                                                  int32_t* __restrict__ row_of,
+                                                                  int32_t* __restrict__ n_total)
+{
+    // [T + T/16] keys, then row_of, one pad word after every 16 (a thread's 16
+    // words start on a different bank for each lane); [T] positions of the
+    // selected tokens; [T] bytes of z
+    extern __shared__ uint32_t stage[];
+    int* pos_st = reinterpret_cast<int*>(stage + T + T / 16 + 1);
+    uint8_t* zst = reinterpret_cast<uint8_t*>(pos_st + T);
+    auto pad = [](int i) { return i + (i >> 4); };
+    __shared__ WarpHist wh;
+    __shared__ int hist[256];
+    __shared__ uint32_t sh_prefix;
+    __shared__ int sh_remaining;
+    __shared__ int sh_warp[32];
+    const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t off = static_cast<int64_t>(b) * T;
+    const int t0 = threadIdx.x * KPT;
+    {
+        float g[KPT];  // all of a thread's loads in flight at once
+#pragma unroll
+        for (int u = 0; u < KPT; ++u) {
+            const int i = threadIdx.x + u * 1024;
+            g[u] = i < T ? p[off + i] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < KPT; ++u) {
+            const int i = threadIdx.x + u * 1024;
+            if (i < T) stage[pad(i)] = gate_key(g[u]);
+        }
+    }
+    __syncthreads();
+    uint32_t key[KPT];
+    bool valid[KPT];
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        valid[u] = t0 + u < T;
+        key[u] = valid[u] ? stage[pad(t0 + u)] : 0u;
+    }
+    // the k-th largest key, as radix_select_kernel finds it
+    const int k_eff = k <= 0 ? 0 : (k >= T ? T : k);
+    uint32_t prefix = 0;
+    int remaining = k;
+    if (k <= 0) {
+        prefix = 0xFFFFFFFFu;
+        remaining = 0;
+    } else if (k >= T) {
+        prefix = 0u;
+        remaining = T;
+    } else {
+        uint32_t mask = 0;
+        for (int shift = 24; shift >= 0; shift -= 8) {
+            hist_clear(wh);
+            __syncthreads();
+#pragma unroll
+            for (int u = 0; u < KPT; ++u) count_key(wh, warp, valid[u] && (key[u] & mask) == prefix, key[u], shift);
+            __syncthreads();
+            hist_sum(wh, hist);
+            __syncthreads();
+            if (warp == 0) hist_pick(hist, remaining, prefix, shift, &sh_prefix, &sh_remaining);
+            __syncthreads();
+            prefix = sh_prefix;
+            remaining = sh_remaining;
+            mask |= 0xFFu << shift;
+            __syncthreads();
+        }
+    }
+    // decisions: above the k-th key, plus the first `remaining` tokens equal to it
+    int neq = 0;
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) neq += (valid[u] && key[u] == prefix) ? 1 : 0;
+    auto block_scan = [&](int v) {  // exclusive scan over the 1024 threads in order
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) sh_warp[warp] = x;
+        __syncthreads();
+        if (warp == 0) {
+            int w = sh_warp[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w += y;
+            }
+            sh_warp[lane] = w - sh_warp[lane];  // exclusive over warps
+        }
+        __syncthreads();
+        const int r = sh_warp[warp] + x - v;
+        __syncthreads();
+        return r;
+    };
+    int eq_rank = block_scan(neq);
+    bool sel[KPT];
+    int nsel = 0;
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        bool take = false;
+        if (valid[u] && key[u] == prefix) {
+            take = eq_rank < remaining;
+            ++eq_rank;
+        }
+        sel[u] = valid[u] && (key[u] > prefix || take);
+        nsel += sel[u];
+    }
+    int lrow = block_scan(nsel);  // its barriers also end every read of the staged keys
+    int* row_st = reinterpret_cast<int*>(stage);
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        if (valid[u]) {
+            zst[t0 + u] = sel[u] ? 1 : 0;
+            row_st[pad(t0 + u)] = sel[u] ? b * k_eff + lrow : -1;
+            if (sel[u]) pos_st[lrow++] = t0 + u;
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < k_eff; i += blockDim.x) pos[static_cast<int64_t>(b) * k_eff + i] = pos_st[i];
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        const int i = threadIdx.x + u * 1024;
+        if (i < T) {
+            z[off + i] = zst[i];
+            row_of[off + i] = row_st[pad(i)];
+        }
+    }
+    if (threadIdx.x == 0) {
+        cu_q[b] = b * k_eff;
+        if (b == B - 1) {
+            cu_q[B] = B * k_eff;
+            *n_total = B * k_eff;
+        }
+    }
 }
 
 struct ChunkCounts {
@@ -305,6 +530,20 @@ extern "C" int logo_select(const float* gate_p, logo_dims dims, int mode, float 
     const int nchunk = (dims.T + kChunk - 1) / kChunk;
     // k = floor(rho * T), with rho read as float32 and the product in double
     const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
+    if (ratio_mode && dims.T <= 16 * 1024) {  // one launch: one block per sequence
+        const int smem =
+            static_cast<int>(round_up((static_cast<size_t>(dims.T) + dims.T / 16 + 1 + dims.T) * 4 + dims.T, 16));
+        if (dims.T <= 4 * 1024) {
+            if (set_smem_limit(select_ratio_small_kernel<4>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
+            select_ratio_small_kernel<4><<<dims.B, 1024, smem, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                     n_sel_total);
+        } else {
+            if (set_smem_limit(select_ratio_small_kernel<16>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
+            select_ratio_small_kernel<16><<<dims.B, 1024, smem, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q,
+                                                                      row_of, n_sel_total);
+        }
+        return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+    }
     if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);
     dim3 grid(nchunk, dims.B);
     count_kernel<<<grid, kThreads, 0, st>>>(gate_p, dims.T, nchunk, ratio_mode, b_th, nullptr, ws.th, ws.counts);

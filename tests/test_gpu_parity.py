@@ -82,6 +82,9 @@ SELECT_CASES = [
     ("normal", 1, 1, 1, 0.0, 1.0),
     ("normal", 1, 1, 0, 0.5, 0.0),
     ("normal", 4, 65536, 1, 0.0, 0.0625),
+    ("ties", 3, 4097, 1, 0.0, 0.25),       # one-block ratio path: 16 tokens per thread, ragged
+    ("ties", 2, 4096, 1, 0.0, 0.25),       # ... 4 tokens per thread, full
+    ("normal", 1, 16385, 1, 0.0, 0.125),   # just past the one-block path
 ]
 
 
