@@ -162,6 +162,15 @@ LAUNCHES_PER_STEP = {"select": 4, "local_fwd": 1, "global_fwd": 3, "combine": 1,
                      "global_bwd": 3, "local_bwd": 3}
 
 
+def launches_per_step(w):
+    """Kernels one step launches: select takes one launch in ratio mode for
+    sequences of at most 16K tokens, four otherwise."""
+    n = sum(LAUNCHES_PER_STEP.values())
+    if w.mode == "ratio" and w.T <= 16384:
+        n -= LAUNCHES_PER_STEP["select"] - 1
+    return n
+
+
 def run_step(layer, g, ev=None):
     """One full step; if ev is given, record an event after each call."""
     from paper_2608_29539_gb300 import logo as L
@@ -550,7 +559,7 @@ def native_arm(a, rank, world, local_rank, dist_on):
             "local_fwd_bwd": {"tflops": fl_local / (l_ms / 1e3) / 1e12, "ms": l_ms},
             "useful_flops_per_step": fl_step, "pairs_per_head": {"local": lp, "global": gp},
             "selected": n, "per_call": breakdown, "roofline": roof,
-            "gpu_launches": sum(LAUNCHES_PER_STEP.values()) * a.steps, "clocks": clk.summary()}
+            "gpu_launches": launches_per_step(w) * a.steps, "clocks": clk.summary()}
 
     # ---- dense comparison: the same global kernels with every token selected
     if not a.no_dense:
