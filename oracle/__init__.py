@@ -84,6 +84,11 @@ def _load():
                                                  _int, _int, _int, _int, _f64p, _f64p]
             lib.oracle_gate.argtypes = [_f32p, _f32p, _i64, _int, _f64p]
             lib.oracle_gate_bwd.argtypes = [_f32p, _f32p, _f32p, _i64, _int, _f64p, _f64p]
+            _i64p = np.ctypeslib.ndpointer(dtype=np.int64, flags="C_CONTIGUOUS")
+            lib.oracle_branch_fwd.argtypes = [_f32p, _int, _int, _i64p, _i64, ctypes.c_void_p, ctypes.c_void_p,
+                                              ctypes.c_void_p, _f64p]
+            lib.oracle_branch_bwd.argtypes = [_f32p, _int, _int, _i64p, _i64, ctypes.c_void_p, ctypes.c_void_p,
+                                              _f32p, _f64p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
             lib.oracle_num_threads.restype = _int
             _lib = lib
     return _lib
@@ -300,3 +305,51 @@ def gate_bwd(x, w, dp):
     if n:
         _load().oracle_gate_bwd(x.reshape(n, dm), _f32(w).reshape(dm), _f32(dp).reshape(n), n, dm, dx, dw)
     return dx.reshape(x.shape), dw
+
+
+def _branch_rows(B, T, rows):
+    if rows is None:
+        return np.arange(B * T, dtype=np.int64)
+    rb, rt = rows
+    return (np.asarray(rb, dtype=np.int64) * T + np.asarray(rt, dtype=np.int64)).reshape(-1)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def branch_fwd(u, A=None, s=None, b=None, rows=None):
+    """Eq. 5 on the rows (row_b, row_t) of u [B, T, H, D] (all rows if None):
+    LP with A [H, D, D], else SO with s, b [H, D].  Returns [nrows, H, D] float64."""
+    u = _f32(u)
+    B, T, H, D = u.shape
+    r = _branch_rows(B, T, rows)
+    A = None if A is None else _f32(A)
+    s = None if s is None else _f32(s)
+    b = None if b is None else _f32(b)
+    g = np.zeros((r.size, H, D), dtype=np.float64)
+    if r.size:
+        _load().oracle_branch_fwd(u, H, D, r, r.size, _ptr(A), _ptr(s), _ptr(b), g)
+    return g
+
+
+def branch_bwd(u, dg, A=None, s=None, rows=None):
+    """Gradients of branch_fwd for dg [nrows, H, D]: (du [nrows, H, D], dA) for LP,
+    (du, ds, db) for SO, float64."""
+    u = _f32(u)
+    B, T, H, D = u.shape
+    r = _branch_rows(B, T, rows)
+    dg = _f32(dg).reshape(r.size, H, D)
+    du = np.zeros((r.size, H, D), dtype=np.float64)
+    if A is not None:
+        A = _f32(A)
+        dA = np.zeros((H, D, D), dtype=np.float64)
+        if r.size:
+            _load().oracle_branch_bwd(u, H, D, r, r.size, _ptr(A), None, dg, du, _ptr(dA), None, None)
+        return du, dA
+    s = _f32(s)
+    ds = np.zeros((H, D), dtype=np.float64)
+    db = np.zeros((H, D), dtype=np.float64)
+    if r.size:
+        _load().oracle_branch_bwd(u, H, D, r, r.size, None, _ptr(s), dg, du, None, _ptr(ds), _ptr(db))
+    return du, ds, db

@@ -66,6 +66,64 @@ void oracle_gate_bwd(const float* x, const float* w, const float* dp, int64_t n,
     }
 }
 
+/* Eq. 5 branch transform U^G_h = phi_{U,h}(U^L_h), for the listed rows r
+ * (indices into the B*T rows of a [B,T,H,D] tensor), in double:
+ *   LP (A != NULL): g[r,h,j] = sum_i u[r,h,i] A[h,i,j]      A [H,D,D]
+ *   SO (A == NULL): g[r,h,j] = u[r,h,j] s[h,j] + b[h,j]      s, b [H,D]
+ * Output g [nrows,H,D]. */
+void oracle_branch_fwd(const float* u, int H, int D, const int64_t* rows, int64_t nrows, const float* A,
+                       const float* s, const float* b, double* g)
+{
+    for (int64_t r = 0; r < nrows; ++r) {
+        for (int h = 0; h < H; ++h) {
+            const float* ur = u + (rows[r] * H + h) * (int64_t)D;
+            double* gr = g + (r * H + h) * (int64_t)D;
+            for (int j = 0; j < D; ++j) {
+                if (A) {
+                    double acc = 0.0;
+                    for (int i = 0; i < D; ++i) acc += (double)ur[i] * (double)A[((int64_t)h * D + i) * D + j];
+                    gr[j] = acc;
+                } else {
+                    gr[j] = (double)ur[j] * (double)s[(int64_t)h * D + j] + (double)b[(int64_t)h * D + j];
+                }
+            }
+        }
+    }
+}
+
+/* Gradients of oracle_branch_fwd for dg [nrows,H,D]:
+ *   LP: du[r,h,i] = sum_j dg[r,h,j] A[h,i,j];  dA[h,i,j] = sum_r u[r,h,i] dg[r,h,j]
+ *   SO: du = dg s;  ds[h,j] = sum_r dg u;  db[h,j] = sum_r dg
+ * Parameter gradients summed over the rows in order. */
+void oracle_branch_bwd(const float* u, int H, int D, const int64_t* rows, int64_t nrows, const float* A,
+                       const float* s, const float* dg, double* du, double* dA, double* ds, double* db)
+{
+    if (A) memset(dA, 0, sizeof(double) * (size_t)H * D * D);
+    else {
+        memset(ds, 0, sizeof(double) * (size_t)H * D);
+        memset(db, 0, sizeof(double) * (size_t)H * D);
+    }
+    for (int64_t r = 0; r < nrows; ++r) {
+        for (int h = 0; h < H; ++h) {
+            const float* ur = u + (rows[r] * H + h) * (int64_t)D;
+            const float* gr = dg + (r * H + h) * (int64_t)D;
+            double* dur = du + (r * H + h) * (int64_t)D;
+            for (int i = 0; i < D; ++i) {
+                if (A) {
+                    double acc = 0.0;
+                    for (int j = 0; j < D; ++j) acc += (double)gr[j] * (double)A[((int64_t)h * D + i) * D + j];
+                    dur[i] = acc;
+                    for (int j = 0; j < D; ++j) dA[((int64_t)h * D + i) * D + j] += (double)ur[i] * (double)gr[j];
+                } else {
+                    dur[i] = (double)gr[i] * (double)s[(int64_t)h * D + i];
+                    ds[(int64_t)h * D + i] += (double)gr[i] * (double)ur[i];
+                    db[(int64_t)h * D + i] += (double)gr[i];
+                }
+            }
+        }
+    }
+}
+
 /* Eq. 3 and Eq. 11 (Sec. 3.2, Budget Control): the realised ratio is
  * F = n_sel / n_valid, and the threshold moves by gamma * sign(F - rho).
  * F and the sign are evaluated in double from the integer counts; b_th and

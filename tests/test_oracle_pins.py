@@ -525,6 +525,58 @@ def test_gate_bwd_matches_torch_autograd_and_finite_differences():
     np.testing.assert_allclose(dwz, (dp.astype(np.float64)[..., None] / 4 * x).sum(axis=(0, 1)), rtol=1e-12)
 
 
+def test_branch_transform_matches_einsum_and_identity():
+    rng = np.random.default_rng(21)
+    u = rng.standard_normal((2, 9, 3, 16)).astype(np.float32)
+    A = rng.standard_normal((3, 16, 16)).astype(np.float32)
+    s_ = rng.standard_normal((3, 16)).astype(np.float32)
+    b_ = rng.standard_normal((3, 16)).astype(np.float32)
+    g = oracle.branch_fwd(u, A=A)
+    ref = np.einsum("bthi,hij->bthj", u.astype(np.float64), A.astype(np.float64)).reshape(-1, 3, 16)
+    np.testing.assert_allclose(g, ref, rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(oracle.branch_fwd(u, s=s_, b=b_),
+                               (u.astype(np.float64) * s_ + b_).reshape(-1, 3, 16), rtol=1e-15, atol=1e-15)
+    # identity initialisation (Sec. 3.2): both forms start as U^G = U^L exactly
+    eye = np.broadcast_to(np.eye(16, dtype=np.float32), (3, 16, 16)).copy()
+    assert (oracle.branch_fwd(u, A=eye) == u.reshape(-1, 3, 16)).all()
+    assert (oracle.branch_fwd(u, s=np.ones((3, 16), np.float32), b=np.zeros((3, 16), np.float32))
+            == u.reshape(-1, 3, 16)).all()
+    # a row subset gives those rows of the full result, in the listed order
+    rb, rt = np.array([1, 0, 1]), np.array([8, 2, 0])
+    np.testing.assert_array_equal(oracle.branch_fwd(u, A=A, rows=(rb, rt)), g.reshape(2, 9, 3, 16)[rb, rt])
+
+
+def test_branch_transform_bwd_matches_torch_autograd():
+    rng = np.random.default_rng(22)
+    u = rng.standard_normal((2, 7, 2, 8)).astype(np.float32)
+    A = rng.standard_normal((2, 8, 8)).astype(np.float32)
+    s_ = rng.standard_normal((2, 8)).astype(np.float32)
+    b_ = rng.standard_normal((2, 8)).astype(np.float32)
+    rb, rt = np.array([0, 0, 1, 1, 1]), np.array([1, 4, 0, 2, 6])
+    dg = rng.standard_normal((5, 2, 8)).astype(np.float32)
+    du, dA = oracle.branch_bwd(u, dg, A=A, rows=(rb, rt))
+    tu = torch.tensor(u, dtype=torch.float64, requires_grad=True)
+    tA = torch.tensor(A, dtype=torch.float64, requires_grad=True)
+    torch.einsum("rhi,hij->rhj", tu[rb, rt], tA).backward(torch.tensor(dg, dtype=torch.float64))
+    np.testing.assert_allclose(du, tu.grad.numpy()[rb, rt], rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(dA, tA.grad.numpy(), rtol=1e-12, atol=1e-13)
+    du2, ds, db = oracle.branch_bwd(u, dg, s=s_, rows=(rb, rt))
+    tu = torch.tensor(u, dtype=torch.float64, requires_grad=True)
+    ts = torch.tensor(s_, dtype=torch.float64, requires_grad=True)
+    tb = torch.tensor(b_, dtype=torch.float64, requires_grad=True)
+    (tu[rb, rt] * ts + tb).backward(torch.tensor(dg, dtype=torch.float64))
+    np.testing.assert_allclose(du2, tu.grad.numpy()[rb, rt], rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(ds, ts.grad.numpy(), rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(db, tb.grad.numpy(), rtol=1e-12, atol=1e-13)
+    # finite difference on one entry of A (the loss is linear in A: exact up to rounding)
+    loss = lambda A_: float((oracle.branch_fwd(u, A=A_, rows=(rb, rt)) * dg.astype(np.float64)).sum())  # noqa: E731
+    hi, lo = A.copy(), A.copy()
+    hi[1, 3, 5] += np.float32(0.5)
+    lo[1, 3, 5] -= np.float32(0.5)
+    step = float(hi[1, 3, 5]) - float(lo[1, 3, 5])
+    assert (loss(hi) - loss(lo)) / step == pytest.approx(dA[1, 3, 5], rel=1e-10, abs=1e-12)
+
+
 def test_ratio_zero_layer_is_pure_local():
     # rho = 0: no token is selected, the layer output is Norm^L(O^L) and no
     # gradient reaches the global branch or the gate.
