@@ -15,6 +15,8 @@
  *   logo_gate_select / logo_gate_bwd
  *                                Eq. 7 gate p = sigmoid(x . w_g) fused ahead of
  *                                logo_select, and its backward
+ *   logo_branch_transform / _bwd Eq. 5 LP / SO transforms U^L -> U^G (Q on the
+ *                                selected rows only)
  *
  * Conventions shared by every entry point
  *   - All tensor pointers are DEVICE pointers owned by the caller.  The
@@ -297,6 +299,42 @@ LOGO_API size_t logo_gate_bwd_workspace_size(logo_dims dims, int d_model);
 LOGO_API int logo_gate_bwd(const logo_bf16* x, const float* w_g, const float* gate_p, const float* dgate_p,
                            int d_model, logo_dims dims, logo_bf16* dx, int accumulate, float* dw_g, void* workspace,
                            size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * logo_branch_transform -- the per-head branch transform of Eq. 5 that turns a
+ *   local-branch tensor into the global branch's, in one of its two forms:
+ *   LP: U^G_h = U^L_h A_h, A [H,D,D] bf16 (A[h][i][j] maps input dimension i to
+ *       output j; identity at initialisation; the paper's default);
+ *   SO: U^G_h = U^L_h * s_h + b_h, s and b [H,D] float32.
+ *   Exactly one form: a_lp, or both s_so and b_so.
+ * Rows: every row when pos is NULL (K and V); otherwise only the packed
+ *   selected rows described by pos / cu_q / n_sel_total (device, from
+ *   logo_select): Q, of which the global branch reads those rows alone.
+ * In : u_l [B,T,H,D] bf16 with H = dims.Hq, the head count of this tensor (Hq
+ *      for Q, Hkv for K and V; dims.Hkv is not read); D 64 or 128; H*D <= 8192.
+ *      LP runs on the tensor cores (warp-level MMA), SO elementwise.
+ * Out: u_g [B,T,H,D] bf16: the listed rows written, other rows untouched.
+ * Errors: LOGO_ERR_INVALID_ARG for a missing or doubled form or pointer;
+ *      LOGO_ERR_UNSUPPORTED for D, H*D or 16-byte alignment. */
+LOGO_API int logo_branch_transform(const logo_bf16* u_l, const logo_bf16* a_lp, const float* s_so, const float* b_so,
+                                   const int32_t* pos, const int32_t* cu_q, const int32_t* n_sel_total,
+                                   logo_bf16* u_g, logo_dims dims, void* stream);
+
+/* logo_branch_transform_bwd -- gradients of logo_branch_transform on the same
+ *   rows, for du_g [B,T,H,D] bf16 (read on the listed rows):
+ *   du_l = du_g A_h^T (LP) or du_g * s_h (SO), written, or added to du_l when
+ *      accumulate = 1 (the caller's gradient of U^L from the local branch);
+ *   LP: da_lp [H,D,D] float32 = sum over the rows of u_l^T du_g;
+ *   SO: ds_so, db_so [H,D] float32 = sums of du_g * u_l and of du_g (either may
+ *      be NULL).  Parameter gradients are summed per block, then over the blocks
+ *      in a fixed order (deterministic).
+ * Workspace: logo_branch_transform_bwd_workspace_size(dims) bytes. */
+LOGO_API size_t logo_branch_transform_bwd_workspace_size(logo_dims dims);
+LOGO_API int logo_branch_transform_bwd(const logo_bf16* u_l, const logo_bf16* a_lp, const float* s_so,
+                                       const int32_t* pos, const int32_t* cu_q, const int32_t* n_sel_total,
+                                       const logo_bf16* du_g, logo_bf16* du_l, int accumulate, float* da_lp,
+                                       float* ds_so, float* db_so, logo_dims dims, void* workspace,
+                                       size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * logo_combine -- ContextNorm per branch (Eq. 9: head-wise RMSNorm over D,

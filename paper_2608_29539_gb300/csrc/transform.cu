@@ -1,0 +1,467 @@
+// transform.cu -- logo_branch_transform / _bwd: the per-head branch transforms
+// of Eq. 5 that turn the local branch's Q/K/V into the global branch's,
+//   LP: U^G_h = U^L_h A_h   (A_h a d x d matrix per head; the paper's default)
+//   SO: U^G_h = U^L_h * s_h + b_h
+// on either every row of a [B, T, H, d] tensor (K and V) or only the packed
+// selected rows (Q: the global branch reads Q^G on those rows alone, so the
+// transform of the other B*T - N rows is never computed).
+//
+// LP is a contraction of 2 d^2 FLOP per row and head against 4 d bytes moved:
+// at d = 128 that is 64 FLOP/byte, more than the CUDA cores can keep up with
+// at HBM speed, so it runs on the tensor cores (warp-level mma.sync over
+// 64-row tiles; per-head operand too small for a tcgen05 tile pipeline to
+// pay).  A block keeps one head's A_h in shared memory and walks a strided
+// share of the row tiles.  The backward computes dU^L = dU^G A_h^T on the same
+// tiles and accumulates dA_h = U^L^T dU^G in registers; per-block partial dA
+// are reduced in block order by a second kernel (deterministic).  SO is
+// elementwise; its ds, db are reduced the same way.
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include "attn_common.cuh"
+#include "host_common.h"
+#include "sm100.cuh"
+
+namespace logo {
+namespace {
+
+constexpr int kTileRows = 64;
+constexpr int kChunksPerHead = 16;  // blocks per head (row tiles strided among them)
+
+// Row r of the listed set -> token index b*T + t (all rows: r itself).
+struct RowSet {
+    const int32_t* pos;    // packed positions, or NULL for every row
+    const int32_t* cu_q;
+    const int32_t* n_sel;  // device count of packed rows
+    int B, T;
+};
+
+__device__ __forceinline__ int row_count(const RowSet& R)
+{
+    return R.pos ? *R.n_sel : R.B * R.T;
+}
+
+__device__ __forceinline__ int64_t row_token(const RowSet& R, int r)
+{
+    if (!R.pos) return r;
+    const int b = seq_of_row(R.cu_q, R.B, r);
+    return static_cast<int64_t>(b) * R.T + R.pos[r];
+}
+
+// [rows][D] bf16 tile in shared memory, 16-byte chunk c of row r stored at
+// chunk c ^ (r & 7): the 8 rows an ldmatrix reads hit 8 different bank groups.
+template <int D>
+__device__ __forceinline__ uint32_t toff(int row, int chunk)
+{
+    return static_cast<uint32_t>(row * (D * 2) + ((chunk ^ (row & 7)) << 4));
+}
+
+// Load rows [0, nrows) of a tile (token indices in tok[]) of head h; rows past
+// the end are zero.
+template <int D>
+__device__ __forceinline__ void load_tile(uint32_t dst, const logo_bf16* src, const int64_t* tok, int nrows, int H,
+                                          int h, int nthreads)
+{
+    constexpr int kChunks = D / 8;
+    for (int idx = threadIdx.x; idx < kTileRows * kChunks; idx += nthreads) {
+        const int r = idx / kChunks, c = idx % kChunks;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (r < nrows) v = *reinterpret_cast<const uint4*>(src + (tok[r] * H + h) * D + c * 8);
+        st_shared_v4(dst + toff<D>(r, c), v.x, v.y, v.z, v.w);
+    }
+}
+
+template <int D>
+__device__ __forceinline__ void load_matrix(uint32_t dst, const logo_bf16* a, int nthreads)
+{
+    constexpr int kChunks = D / 8;
+    for (int idx = threadIdx.x; idx < D * kChunks; idx += nthreads) {
+        const int r = idx / kChunks, c = idx % kChunks;
+        const uint4 v = *reinterpret_cast<const uint4*>(a + r * D + c * 8);
+        st_shared_v4(dst + toff<D>(r, c), v.x, v.y, v.z, v.w);
+    }
+}
+
+// LP forward: u_g[row] = u_l[row] A_h.  4 warps, 16 rows of the 64-row tile each.
+template <int D>
+__global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict__ u_l,
+                                                     const logo_bf16* __restrict__ a, RowSet R, int H,
+                                                     logo_bf16* __restrict__ u_g)
+{
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ int64_t tok[kTileRows];
+    const uint32_t sA = smem_u32(smem), sU = sA + D * D * 2;
+    const int h = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mi = lane >> 3, rr = lane & 7, gid = lane >> 2, tig = lane & 3;
+    load_matrix<D>(sA, a + static_cast<int64_t>(h) * D * D, 128);
+    const int n = row_count(R);
+    const int ntiles = (n + kTileRows - 1) / kTileRows;
+    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int r0 = tile * kTileRows, nr = min(kTileRows, n - r0);
+        if (threadIdx.x < kTileRows) tok[threadIdx.x] = threadIdx.x < nr ? row_token(R, r0 + threadIdx.x) : 0;
+        __syncthreads();
+        load_tile<D>(sU, u_l, tok, nr, H, h, 128);
+        __syncthreads();
+        float acc[D / 8][4];
+#pragma unroll
+        for (int nt = 0; nt < D / 8; ++nt)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[nt][i] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+            uint32_t fa[4];
+            ldsm_x4(sU + toff<D>(warp * 16 + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), fa[0], fa[1], fa[2], fa[3]);
+#pragma unroll
+            for (int np = 0; np < D / 16; ++np) {
+                uint32_t b0, b1, b2, b3;  // A_h rows k (input dim), columns n (output dim)
+                ldsm_x4_trans(sA + toff<D>(16 * ks + (mi & 1) * 8 + rr, 2 * np + (mi >> 1)), b0, b1, b2, b3);
+                mma_bf16_16816(acc[2 * np], fa, b0, b1);
+                mma_bf16_16816(acc[2 * np + 1], fa, b2, b3);
+            }
+        }
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int r = warp * 16 + gid + half * 8;
+            if (r < nr) {
+                logo_bf16* dst = u_g + (tok[r] * H + h) * D + 2 * tig;
+#pragma unroll
+                for (int nt = 0; nt < D / 8; ++nt)
+                    *reinterpret_cast<uint32_t*>(dst + nt * 8) = pack_bf16x2(acc[nt][2 * half], acc[nt][2 * half + 1]);
+            }
+        }
+        __syncthreads();
+    }
+}
+
+// LP backward: du_l[row] (+)= du_g[row] A_h^T, and dA_h += u_l^T du_g over the
+// block's rows.  D/16 warps: for dU, warp w takes rows 16 (w % 4).. and output
+// columns 64 (w / 4)..; for dA, rows 16w.. of the D x D result.
+// part: [H][gridDim.x][D][D] float32.
+template <int D>
+__global__ void __launch_bounds__(D * 2) lp_bwd_kernel(const logo_bf16* __restrict__ u_l,
+                                                       const logo_bf16* __restrict__ a,
+                                                       const logo_bf16* __restrict__ du_g, RowSet R, int H,
+                                                       logo_bf16* __restrict__ du_l, int accumulate,
+                                                       float* __restrict__ part)
+{
+    constexpr int kThreads = D * 2;
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ int64_t tok[kTileRows];
+    const uint32_t sA = smem_u32(smem), sU = sA + D * D * 2, sG = sU + kTileRows * D * 2;
+    const int h = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int mi = lane >> 3, rr = lane & 7, gid = lane >> 2, tig = lane & 3;
+    load_matrix<D>(sA, a + static_cast<int64_t>(h) * D * D, kThreads);
+    float acc_a[D / 8][4];
+#pragma unroll
+    for (int nt = 0; nt < D / 8; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc_a[nt][i] = 0.f;
+    const int n = row_count(R);
+    const int ntiles = (n + kTileRows - 1) / kTileRows;
+    const int rg = warp & 3, cb = (warp >> 2) * 64;  // dU: row group and first output column
+    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int r0 = tile * kTileRows, nr = min(kTileRows, n - r0);
+        if (threadIdx.x < kTileRows) tok[threadIdx.x] = threadIdx.x < nr ? row_token(R, r0 + threadIdx.x) : 0;
+        __syncthreads();
+        load_tile<D>(sU, u_l, tok, nr, H, h, kThreads);
+        load_tile<D>(sG, du_g, tok, nr, H, h, kThreads);
+        __syncthreads();
+        // dU = dG A^T: rows 16 rg.., output columns cb .. cb + 63 (A_h rows i)
+        {
+            float acc[8][4];
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) acc[nt][i] = 0.f;
+#pragma unroll
+            for (int ks = 0; ks < D / 16; ++ks) {  // k: A_h columns j
+                uint32_t fa[4];
+                ldsm_x4(sG + toff<D>(rg * 16 + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), fa[0], fa[1], fa[2], fa[3]);
+#pragma unroll
+                for (int np = 0; np < 4; ++np) {
+                    uint32_t b0, b1, b2, b3;  // B(k = j, n = i) = A_h[i][j]: rows n, k contiguous
+                    ldsm_x4(sA + toff<D>(cb + np * 16 + (mi >> 1) * 8 + rr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
+                    mma_bf16_16816(acc[2 * np], fa, b0, b1);
+                    mma_bf16_16816(acc[2 * np + 1], fa, b2, b3);
+                }
+            }
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int r = rg * 16 + gid + half * 8;
+                if (r < nr) {
+                    logo_bf16* dst = du_l + (tok[r] * H + h) * D + cb + 2 * tig;
+#pragma unroll
+                    for (int nt = 0; nt < 8; ++nt) {
+                        float x0 = acc[nt][2 * half], x1 = acc[nt][2 * half + 1];
+                        uint32_t* p = reinterpret_cast<uint32_t*>(dst + nt * 8);
+                        if (accumulate) {
+                            const float2 old = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+                            x0 += old.x;
+                            x1 += old.y;
+                        }
+                        *p = pack_bf16x2(x0, x1);
+                    }
+                }
+            }
+        }
+        // dA += U^T dG: result rows i = 16 warp .., all columns j; k = the tile's rows
+#pragma unroll
+        for (int ks = 0; ks < kTileRows / 16; ++ks) {
+            uint32_t fa[4];  // A(m = i, k = r) = U[r][i]: stored rows k, m contiguous
+            ldsm_x4_trans(sU + toff<D>(16 * ks + (mi >> 1) * 8 + rr, 2 * warp + (mi & 1)), fa[0], fa[1], fa[2], fa[3]);
+#pragma unroll
+            for (int np = 0; np < D / 16; ++np) {
+                uint32_t b0, b1, b2, b3;  // B(k = r, n = j) = dG[r][j]
+                ldsm_x4_trans(sG + toff<D>(16 * ks + (mi & 1) * 8 + rr, 2 * np + (mi >> 1)), b0, b1, b2, b3);
+                mma_bf16_16816(acc_a[2 * np], fa, b0, b1);
+                mma_bf16_16816(acc_a[2 * np + 1], fa, b2, b3);
+            }
+        }
+        __syncthreads();
+    }
+    float* pp = part + (static_cast<int64_t>(h) * gridDim.x + blockIdx.x) * D * D;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        const int i = warp * 16 + gid + half * 8;
+#pragma unroll
+        for (int nt = 0; nt < D / 8; ++nt) {
+            pp[i * D + nt * 8 + 2 * tig] = acc_a[nt][2 * half];
+            pp[i * D + nt * 8 + 2 * tig + 1] = acc_a[nt][2 * half + 1];
+        }
+    }
+}
+
+// out[h][e] = sum over c (in order) of part[h][c][e], e < per_head.
+__global__ void __launch_bounds__(256) reduce_parts_kernel(const float* __restrict__ part, int nchunk, int per_head,
+                                                           int H, float* __restrict__ out)
+{
+    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (e >= static_cast<int64_t>(H) * per_head) return;
+    const int h = static_cast<int>(e / per_head), x = static_cast<int>(e % per_head);
+    float s = 0.f;
+    for (int c = 0; c < nchunk; ++c) s += part[(static_cast<int64_t>(h) * nchunk + c) * per_head + x];
+    out[e] = s;
+}
+
+// SO forward: u_g = u_l * s + b on the listed rows; a thread per 8-element vector.
+__global__ void __launch_bounds__(256) so_fwd_kernel(const logo_bf16* __restrict__ u_l, const float* __restrict__ s,
+                                                     const float* __restrict__ b, RowSet R, int H, int D,
+                                                     logo_bf16* __restrict__ u_g)
+{
+    const int nvec = H * D / 8;
+    const int64_t total = static_cast<int64_t>(row_count(R)) * nvec;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int r = static_cast<int>(i / nvec), v = static_cast<int>(i % nvec);
+        const int64_t off = row_token(R, r) * H * D + v * 8;
+        const uint4 raw = *reinterpret_cast<const uint4*>(u_l + off);
+        const __nv_bfloat162* x = reinterpret_cast<const __nv_bfloat162*>(&raw);
+        uint4 o;
+        uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float2 f = __bfloat1622float2(x[q]);
+            const int e = v * 8 + 2 * q;
+            ow[q] = pack_bf16x2(fmaf(f.x, s[e], b[e]), fmaf(f.y, s[e + 1], b[e + 1]));
+        }
+        *reinterpret_cast<uint4*>(u_g + off) = o;
+    }
+}
+
+// SO backward: du_l (+)= du_g * s; ds += du_g * u_l, db += du_g.  A thread owns
+// fixed vectors (VPT of them) of the [H, D] row for all rows of its block.
+// part: [gridDim.x][2][H*D] float32 (ds, db).
+template <int VPT>
+__global__ void __launch_bounds__(256) so_bwd_kernel(const logo_bf16* __restrict__ u_l, const float* __restrict__ s,
+                                                     const logo_bf16* __restrict__ du_g, RowSet R, int H, int D,
+                                                     logo_bf16* __restrict__ du_l, int accumulate,
+                                                     float* __restrict__ part)
+{
+    const int nvec = H * D / 8;
+    float acc_s[VPT][8], acc_b[VPT][8];
+#pragma unroll
+    for (int k = 0; k < VPT; ++k)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc_s[k][i] = acc_b[k][i] = 0.f;
+    const int n = row_count(R);
+    for (int r = blockIdx.x; r < n; r += gridDim.x) {
+        const int64_t base = row_token(R, r) * H * D;
+#pragma unroll
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * 256;
+            if (v >= nvec) continue;
+            const uint4 gu = *reinterpret_cast<const uint4*>(du_g + base + v * 8);
+            const uint4 uu = *reinterpret_cast<const uint4*>(u_l + base + v * 8);
+            const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&gu);
+            const __nv_bfloat162* u2 = reinterpret_cast<const __nv_bfloat162*>(&uu);
+            uint4 prev = make_uint4(0u, 0u, 0u, 0u);
+            if (accumulate) prev = *reinterpret_cast<const uint4*>(du_l + base + v * 8);
+            const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&prev);
+            uint4 o;
+            uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float2 g = __bfloat1622float2(g2[q]), u = __bfloat1622float2(u2[q]);
+                const int e = v * 8 + 2 * q;
+                float x0 = g.x * s[e], x1 = g.y * s[e + 1];
+                if (accumulate) {
+                    const float2 pv = __bfloat1622float2(p2[q]);
+                    x0 += pv.x;
+                    x1 += pv.y;
+                }
+                ow[q] = pack_bf16x2(x0, x1);
+                acc_s[k][2 * q] = fmaf(g.x, u.x, acc_s[k][2 * q]);
+                acc_s[k][2 * q + 1] = fmaf(g.y, u.y, acc_s[k][2 * q + 1]);
+                acc_b[k][2 * q] += g.x;
+                acc_b[k][2 * q + 1] += g.y;
+            }
+            *reinterpret_cast<uint4*>(du_l + base + v * 8) = o;
+        }
+    }
+    const int64_t hd = static_cast<int64_t>(H) * D;
+#pragma unroll
+    for (int k = 0; k < VPT; ++k) {
+        const int v = threadIdx.x + k * 256;
+        if (v >= nvec) continue;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            part[static_cast<int64_t>(blockIdx.x) * 2 * hd + v * 8 + i] = acc_s[k][i];
+            part[static_cast<int64_t>(blockIdx.x) * 2 * hd + hd + v * 8 + i] = acc_b[k][i];
+        }
+    }
+}
+
+// ds / db from the [grid][2][H*D] parts (block order).
+__global__ void __launch_bounds__(256) so_reduce_kernel(const float* __restrict__ part, int nblk, int hd,
+                                                        float* __restrict__ ds, float* __restrict__ db)
+{
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= 2 * hd) return;
+    const int w = e / hd, x = e % hd;
+    float s = 0.f;
+    for (int b = 0; b < nblk; ++b) s += part[(static_cast<int64_t>(b) * 2 + w) * hd + x];
+    float* dst = w == 0 ? ds : db;
+    if (dst) dst[x] = s;
+}
+
+int so_vpt(const logo_dims& d)
+{
+    const int nvec = d.Hq * d.D / 8;
+    const int need = (nvec + 255) / 256;
+    return need <= 1 ? 1 : need <= 2 ? 2 : 4;
+}
+
+int so_bwd_blocks(const logo_dims& d)
+{
+    const int64_t rows = static_cast<int64_t>(d.B) * d.T;
+    const int64_t cap = static_cast<int64_t>(device_sm_count()) * 4;
+    return static_cast<int>(rows < cap ? rows : cap);
+}
+
+int check_transform(const logo_dims& d, const void* u, const void* out)
+{
+    if (d.B < 1 || d.T < 1 || d.Hq < 1) return LOGO_ERR_INVALID_ARG;
+    if (d.D != 64 && d.D != 128) return LOGO_ERR_UNSUPPORTED;
+    if (static_cast<int64_t>(d.B) * d.T > (1ll << 30)) return LOGO_ERR_UNSUPPORTED;
+    if (d.Hq * d.D > 8192) return LOGO_ERR_UNSUPPORTED;
+    if (!aligned16(u) || !aligned16(out)) return LOGO_ERR_UNSUPPORTED;
+    return LOGO_OK;
+}
+
+template <int D>
+int launch_lp_fwd(const logo_bf16* u_l, const logo_bf16* a, const RowSet& R, int H, logo_bf16* u_g,
+                  cudaStream_t st)
+{
+    const int smem = D * D * 2 + kTileRows * D * 2;
+    if (set_smem_limit(lp_fwd_kernel<D>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
+    lp_fwd_kernel<D><<<dim3(kChunksPerHead, H), 128, smem, st>>>(u_l, a, R, H, u_g);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+template <int D>
+int launch_lp_bwd(const logo_bf16* u_l, const logo_bf16* a, const logo_bf16* du_g, const RowSet& R, int H,
+                  logo_bf16* du_l, int accumulate, float* da, float* part, cudaStream_t st)
+{
+    const int smem = D * D * 2 + 2 * kTileRows * D * 2;
+    if (set_smem_limit(lp_bwd_kernel<D>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
+    lp_bwd_kernel<D><<<dim3(kChunksPerHead, H), D * 2, smem, st>>>(u_l, a, du_g, R, H, du_l, accumulate, part);
+    if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    const int64_t total = static_cast<int64_t>(H) * D * D;
+    reduce_parts_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(part, kChunksPerHead, D * D, H,
+                                                                                   da);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace logo
+
+using namespace logo;
+
+extern "C" int logo_branch_transform(const logo_bf16* u_l, const logo_bf16* a_lp, const float* s_so,
+                                     const float* b_so, const int32_t* pos, const int32_t* cu_q,
+                                     const int32_t* n_sel_total, logo_bf16* u_g, logo_dims dims, void* stream)
+{
+    int rc = check_transform(dims, u_l, u_g);
+    if (rc != LOGO_OK) return rc;
+    if (!u_l || !u_g) return LOGO_ERR_INVALID_ARG;
+    if ((a_lp != nullptr) == (s_so != nullptr || b_so != nullptr)) return LOGO_ERR_INVALID_ARG;  // exactly one form
+    if (!a_lp && (!s_so || !b_so)) return LOGO_ERR_INVALID_ARG;
+    if (pos && (!cu_q || !n_sel_total)) return LOGO_ERR_INVALID_ARG;
+    if (a_lp && !aligned16(a_lp)) return LOGO_ERR_UNSUPPORTED;
+    const RowSet R{pos, cu_q, n_sel_total, dims.B, dims.T};
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (a_lp) {
+        return dims.D == 128 ? launch_lp_fwd<128>(u_l, a_lp, R, dims.Hq, u_g, st)
+                             : launch_lp_fwd<64>(u_l, a_lp, R, dims.Hq, u_g, st);
+    }
+    const int64_t work = static_cast<int64_t>(dims.B) * dims.T * dims.Hq * dims.D / 8;
+    const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
+    const int64_t blocks = (work + 255) / 256;
+    so_fwd_kernel<<<static_cast<unsigned>(blocks < cap ? blocks : cap), 256, 0, st>>>(u_l, s_so, b_so, R, dims.Hq,
+                                                                                       dims.D, u_g);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
+extern "C" size_t logo_branch_transform_bwd_workspace_size(logo_dims dims)
+{
+    if (dims.B < 1 || dims.T < 1 || dims.Hq < 1 || (dims.D != 64 && dims.D != 128) || dims.Hq * dims.D > 8192)
+        return 0;
+    const size_t lp = static_cast<size_t>(dims.Hq) * kChunksPerHead * dims.D * dims.D * sizeof(float);
+    const size_t so = static_cast<size_t>(so_bwd_blocks(dims)) * 2 * dims.Hq * dims.D * sizeof(float);
+    return lp > so ? lp : so;
+}
+
+extern "C" int logo_branch_transform_bwd(const logo_bf16* u_l, const logo_bf16* a_lp, const float* s_so,
+                                         const int32_t* pos, const int32_t* cu_q, const int32_t* n_sel_total,
+                                         const logo_bf16* du_g, logo_bf16* du_l, int accumulate, float* da_lp,
+                                         float* ds_so, float* db_so, logo_dims dims, void* workspace,
+                                         size_t workspace_bytes, void* stream)
+{
+    int rc = check_transform(dims, u_l, du_l);
+    if (rc != LOGO_OK) return rc;
+    if (!u_l || !du_g || !du_l) return LOGO_ERR_INVALID_ARG;
+    if ((a_lp != nullptr) == (s_so != nullptr)) return LOGO_ERR_INVALID_ARG;  // exactly one form
+    if (a_lp && !da_lp) return LOGO_ERR_INVALID_ARG;
+    if (accumulate != 0 && accumulate != 1) return LOGO_ERR_INVALID_ARG;
+    if (pos && (!cu_q || !n_sel_total)) return LOGO_ERR_INVALID_ARG;
+    if (!aligned16(du_g) || (a_lp && !aligned16(a_lp))) return LOGO_ERR_UNSUPPORTED;
+    if (!workspace || workspace_bytes < logo_branch_transform_bwd_workspace_size(dims)) return LOGO_ERR_WORKSPACE;
+    const RowSet R{pos, cu_q, n_sel_total, dims.B, dims.T};
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    float* part = static_cast<float*>(workspace);
+    if (a_lp) {
+        return dims.D == 128 ? launch_lp_bwd<128>(u_l, a_lp, du_g, R, dims.Hq, du_l, accumulate, da_lp, part, st)
+                             : launch_lp_bwd<64>(u_l, a_lp, du_g, R, dims.Hq, du_l, accumulate, da_lp, part, st);
+    }
+    const int grid = so_bwd_blocks(dims);
+    switch (so_vpt(dims)) {
+        case 1: so_bwd_kernel<1><<<grid, 256, 0, st>>>(u_l, s_so, du_g, R, dims.Hq, dims.D, du_l, accumulate, part); break;
+        case 2: so_bwd_kernel<2><<<grid, 256, 0, st>>>(u_l, s_so, du_g, R, dims.Hq, dims.D, du_l, accumulate, part); break;
+        default: so_bwd_kernel<4><<<grid, 256, 0, st>>>(u_l, s_so, du_g, R, dims.Hq, dims.D, du_l, accumulate, part); break;
+    }
+    if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    const int hd = dims.Hq * dims.D;
+    so_reduce_kernel<<<(2 * hd + 255) / 256, 256, 0, st>>>(part, grid, hd, ds_so, db_so);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}

@@ -60,6 +60,10 @@ _SIGS = {
     "logo_gate_select": (_c_int, [_vp, _vp, _c_int, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp,
                                   _vp, _c_size, _vp]),
     "logo_gate_bwd_workspace_size": (_c_size, [Dims, _c_int]),
+    "logo_branch_transform": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, Dims, _vp]),
+    "logo_branch_transform_bwd_workspace_size": (_c_size, [Dims]),
+    "logo_branch_transform_bwd": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_int, _vp, _vp, _vp, Dims, _vp,
+                                           _c_size, _vp]),
     "logo_gate_bwd": (_c_int, [_vp, _vp, _vp, _vp, _c_int, Dims, _vp, _c_int, _vp, _vp, _c_size, _vp]),
     "logo_select_noalloc": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp]),
     "logo_select_device_threshold": (_c_int, [_vp, Dims, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
@@ -228,6 +232,49 @@ def logo_gate_bwd(x, w_g, gate_p, dgate_p, dx=None, accumulate: bool = False, dw
     _call("logo_gate_bwd", _p(x), _p(w_g), _p(gate_p), _p(dgate_p), int(dm), dims, _p(dx), int(bool(accumulate)),
           _p(dw_g), _p(ws), nbytes, _stream())
     return dx, dw_g
+
+
+def _transform_rows(rows):
+    if rows is None:
+        return None, None, None
+    pos, cu_q, n_sel_total = rows
+    return pos, cu_q, n_sel_total
+
+
+def logo_branch_transform(u_l, a=None, s=None, b=None, rows=None, u_g=None):
+    """Eq. 5: U^G = U^L A (LP, a [H, D, D] bf16) or U^L * s + b (SO, s and b
+    [H, D] float32), on every row, or on the packed selected rows when rows =
+    (pos, cu_q, n_sel_total).  u_l [B, T, H, D] bf16.  Returns u_g."""
+    _need(u_l, torch.bfloat16, "u_l")
+    B, T, H, D = u_l.shape
+    u_g = u_g if u_g is not None else torch.empty_like(u_l)
+    pos, cu_q, n_sel = _transform_rows(rows)
+    _call("logo_branch_transform", _p(u_l), _p(a), _p(s), _p(b), _p(pos), _p(cu_q), _p(n_sel), _p(u_g),
+          Dims(B, T, H, H, D), _stream())
+    return u_g
+
+
+def logo_branch_transform_bwd(u_l, du_g, a=None, s=None, rows=None, du_l=None, accumulate: bool = False,
+                              workspace=None):
+    """Gradients of logo_branch_transform.  Returns (du_l, da) for LP and
+    (du_l, ds, db) for SO."""
+    _need(u_l, torch.bfloat16, "u_l")
+    B, T, H, D = u_l.shape
+    dev = u_l.device
+    dims = Dims(B, T, H, H, D)
+    if du_l is None:
+        if accumulate:
+            raise ValueError("accumulate needs the du_l to add to")
+        du_l = torch.empty_like(u_l)
+    da = torch.empty((H, D, D), dtype=torch.float32, device=dev) if a is not None else None
+    ds = torch.empty((H, D), dtype=torch.float32, device=dev) if a is None else None
+    db = torch.empty((H, D), dtype=torch.float32, device=dev) if a is None else None
+    nbytes = int(lib().logo_branch_transform_bwd_workspace_size(dims))
+    ws = _workspace(nbytes, dev, workspace)
+    pos, cu_q, n_sel = _transform_rows(rows)
+    _call("logo_branch_transform_bwd", _p(u_l), _p(a), _p(s), _p(pos), _p(cu_q), _p(n_sel), _p(du_g), _p(du_l),
+          int(bool(accumulate)), _p(da), _p(ds), _p(db), dims, _p(ws), nbytes, _stream())
+    return (du_l, da) if a is not None else (du_l, ds, db)
 
 
 def logo_select_device_threshold(gate_p, b_th, z=None, pos=None, cu_q=None, row_of=None, n_sel_total=None,

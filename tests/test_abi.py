@@ -178,6 +178,33 @@ def test_gate_host_checks(lib):
     assert bwd(odd, 0, null, null, 0) == logo.LOGO_ERR_UNSUPPORTED
 
 
+def test_branch_transform_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = logo.lib()
+    d = logo.Dims(2, 300, 4, 4, 128)
+    null = None
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected before use
+    odd = ctypes.c_void_p((1 << 20) + 2)
+    fwd = lambda u, a, s_, b, pos, cu, n, out, dims: L.logo_branch_transform(u, a, s_, b, pos, cu, n, out, dims,  # noqa: E731
+                                                                              null)
+    assert fwd(fake, null, null, null, null, null, null, fake, d) == logo.LOGO_ERR_INVALID_ARG       # no form
+    assert fwd(fake, fake, fake, fake, null, null, null, fake, d) == logo.LOGO_ERR_INVALID_ARG       # both forms
+    assert fwd(fake, null, fake, null, null, null, null, fake, d) == logo.LOGO_ERR_INVALID_ARG       # SO without b
+    assert fwd(fake, fake, null, null, fake, null, fake, fake, d) == logo.LOGO_ERR_INVALID_ARG       # rows without cu_q
+    assert fwd(fake, fake, null, null, null, null, null, fake, logo.Dims(2, 300, 4, 4, 96)) == logo.LOGO_ERR_UNSUPPORTED
+    assert fwd(fake, fake, null, null, null, null, null, fake, logo.Dims(2, 300, 72, 72, 128)) == logo.LOGO_ERR_UNSUPPORTED
+    assert fwd(odd, fake, null, null, null, null, null, fake, d) == logo.LOGO_ERR_UNSUPPORTED
+    ws = L.logo_branch_transform_bwd_workspace_size(d)
+    assert ws >= 4 * 128 * 128 * 4
+    bwd = lambda a, s_, acc, da, w, wb: L.logo_branch_transform_bwd(fake, a, s_, null, null, null, fake, fake, acc,  # noqa: E731
+                                                                    da, null, null, d, w, wb, null)
+    assert bwd(fake, fake, 0, fake, fake, ws) == logo.LOGO_ERR_INVALID_ARG   # both forms
+    assert bwd(fake, null, 0, null, fake, ws) == logo.LOGO_ERR_INVALID_ARG   # LP without da
+    assert bwd(fake, null, 3, fake, fake, ws) == logo.LOGO_ERR_INVALID_ARG   # accumulate flag
+    assert bwd(fake, null, 0, fake, fake, ws - 4) == logo.LOGO_ERR_WORKSPACE
+    assert bwd(fake, null, 0, fake, null, ws) == logo.LOGO_ERR_WORKSPACE
+
+
 def test_workspace_sizes_grow_with_shape(lib):
     from paper_2608_29539_gb300 import logo
     L = logo.lib()
