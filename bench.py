@@ -424,6 +424,29 @@ def fusions_bench(layer, x, w, dev, pk):
     byts = 3 * ntok * tok_row + 2 * n * tok_row
     out["combine_bwd_gains"] = {"ms": ms_g, "ms_without_gains": ms_p, "GB_per_s": byts / ms_g / 1e6,
                                 "frac_of_hbm_peak": byts / ms_g / 1e6 / pk["hbm"], "bytes": byts, "launches": 2}
+    # Eq. 5 LP transforms: Q^G on the selected rows only, K^G on every row, and
+    # the backward of the K transform (dK^L accumulated, dA)
+    A = (torch.randn((w.Hkv, w.D, w.D), generator=g, device=dev) / w.D ** 0.5).to(torch.bfloat16)
+    Aq = (torch.randn((w.Hq, w.D, w.D), generator=g, device=dev) / w.D ** 0.5).to(torch.bfloat16)
+    qg, kg = torch.empty_like(x["qL"]), torch.empty_like(x["kL"])
+    dkl = torch.zeros_like(x["kL"])
+    tws = torch.empty((int(L.lib().logo_branch_transform_bwd_workspace_size(
+        L.Dims(w.B, w.T, w.Hkv, w.Hkv, w.D))),), dtype=torch.uint8, device=dev)
+    rows = (layer.pos, layer.cu_q, layer.n_sel)
+    lp_q = lambda: L.logo_branch_transform(x["qL"], a=Aq, rows=rows, u_g=qg)  # noqa: E731
+    lp_k = lambda: L.logo_branch_transform(x["kL"], a=A, u_g=kg)  # noqa: E731
+    dkg = x["dO"][:, :, :w.Hkv].contiguous()  # a stand-in dK^G of the right shape
+    lp_kb = lambda: L.logo_branch_transform_bwd(x["kL"], dkg, a=A, du_l=dkl, accumulate=True,  # noqa: E731
+                                                workspace=tws)
+    kv_row = w.Hkv * w.D * 2
+    for name, fn, rows_n, row_b, heads, passes in (("lp_q_selected_rows", lp_q, n, tok_row, w.Hq, 2),
+                                                   ("lp_k_all_rows", lp_k, ntok, kv_row, w.Hkv, 2),
+                                                   ("lp_k_backward", lp_kb, ntok, kv_row, w.Hkv, 4)):
+        ms = timed(fn)
+        byts = passes * rows_n * row_b
+        fl = (2 if passes == 2 else 4) * rows_n * heads * w.D * w.D
+        out[name] = {"ms": ms, "rows": rows_n, "GB_per_s": byts / ms / 1e6,
+                     "frac_of_hbm_peak": byts / ms / 1e6 / pk["hbm"], "tflops": fl / ms / 1e9, "bytes": byts}
     return out
 
 

@@ -3,9 +3,13 @@ C-ABI entry points (forward: select, local, global, combine; backward:
 combine_bwd, global_bwd, local_bwd).  Buffers and workspaces are allocated
 once per shape and reused, so a step launches kernels only.
 
-The caller owns everything outside the path: the projections of Eq. 4/5, the
-gate logits and their sigmoid (Eq. 7), the output projection, and the chain
-rule through the sigmoid for ``dgate_p``.
+`forward` / `backward` take the branch inputs and the gate values as the
+caller made them (the projections of Eq. 4/5, the gate of Eq. 7 and the
+output projection stay outside).  `forward_fused` / `backward_fused` also
+run the gate of Eq. 7 from the layer input, the Eq. 5 branch transforms
+(Q^G on the selected rows only) and the ContextNorm gain gradients, so the
+caller passes x, w_g, Q^L/K^L/V^L and the transform parameters, and gets back
+every gradient of those.
 """
 from __future__ import annotations
 
@@ -89,4 +93,53 @@ class LogoAttention:
         L.logo_local_attn_bwd(qL, kL, vL, self.o_l, self.lse_l, self.dO_l, c.window, c.scale, self.dqL, self.dkL,
                               self.dvL, workspace=self.ws)
         return dict(dqL=self.dqL, dkL=self.dkL, dvL=self.dvL, dqG=self.dqG, dkG=self.dkG, dvG=self.dvG,
+                    dgate_p=self.dgate)
+
+    # ------------------------------------------------------------ fused path
+    def forward_fused(self, x, w_g, qL, kL, vL, tq, tk, tv, gain_l=None, gain_g=None):
+        """Eq. 7 gate + select, Eq. 5 transforms, both branches, Eq. 9/10.
+
+        x [B, T, d_model] bf16 and w_g [d_model] float32 feed the gate; tq, tk,
+        tv are the Eq. 5 parameters of Q, K, V: a dict {"a": [H, D, D] bf16}
+        (LP) or {"s": [H, D], "b": [H, D] float32} (SO).  Returns o."""
+        c = self.cfg
+        if not hasattr(self, "gate_p"):
+            self.gate_p = torch.empty((c.B, c.T), dtype=torch.float32, device=qL.device)
+            self.qG = torch.empty_like(qL)
+            self.kG = torch.empty_like(kL)
+            self.vG = torch.empty_like(vL)
+        L.logo_gate_select(x, w_g, c.mode, c.b_th, c.ratio, self.gate_p, self.z, self.pos, self.cu_q, self.row_of,
+                           self.n_sel, workspace=self.ws)
+        rows = (self.pos, self.cu_q, self.n_sel)
+        L.logo_branch_transform(qL, rows=rows, u_g=self.qG, **tq)  # Q^G on the selected rows only
+        L.logo_branch_transform(kL, u_g=self.kG, **tk)
+        L.logo_branch_transform(vL, u_g=self.vG, **tv)
+        return self.forward(qL, kL, vL, self.qG, self.kG, self.vG, self.gate_p, gain_l, gain_g)
+
+    def backward_fused(self, dO, x, w_g, qL, kL, vL, tq, tk, tv, gain_l=None, gain_g=None):
+        """Gradients of forward_fused: dqL/dkL/dvL (local branch plus the
+        transforms' share of the global one), the transform parameters (dA or
+        ds/db for q, k, v), the ContextNorm gains, x (the gate's share) and w_g."""
+        c = self.cfg
+        if not hasattr(self, "dgain_l"):
+            self.dgain_l = torch.empty((c.Hq, c.D), dtype=torch.float32, device=dO.device)
+            self.dgain_g = torch.empty_like(self.dgain_l)
+            self.dx = torch.empty_like(x)
+            self.dw_g = torch.empty_like(w_g)
+        L.logo_combine_bwd_gains(dO, self.o_l, self.o_c, self.gate_p, self.z, self.row_of, gain_l, gain_g, c.eps,
+                                 self.dO_l, self.dO_c, self.dgate, self.dgain_l, self.dgain_g)
+        L.logo_global_sparse_attn_bwd(self.qG, self.kG, self.vG, self.pos, self.cu_q, self.n_sel, self.o_c,
+                                      self.lse_c, self.dO_c, c.scale, self.dqG, self.dkG, self.dvG,
+                                      workspace=self.ws)
+        L.logo_local_attn_bwd(qL, kL, vL, self.o_l, self.lse_l, self.dO_l, c.window, c.scale, self.dqL, self.dkL,
+                              self.dvL, workspace=self.ws)
+        rows = (self.pos, self.cu_q, self.n_sel)
+        back = lambda t: {k: v for k, v in t.items() if k != "b"}  # noqa: E731  (b does not enter the backward)
+        tqg = L.logo_branch_transform_bwd(qL, self.dqG, rows=rows, du_l=self.dqL, accumulate=True, **back(tq))
+        tkg = L.logo_branch_transform_bwd(kL, self.dkG, du_l=self.dkL, accumulate=True, **back(tk))
+        tvg = L.logo_branch_transform_bwd(vL, self.dvG, du_l=self.dvL, accumulate=True, **back(tv))
+        L.logo_gate_bwd(x, w_g, self.gate_p, self.dgate, dx=self.dx, dw_g=self.dw_g)
+        names = lambda t, g: ({"dA": g[1]} if "a" in t else {"ds": g[1], "db": g[2]})  # noqa: E731
+        return dict(dqL=self.dqL, dkL=self.dkL, dvL=self.dvL, tq=names(tq, tqg), tk=names(tk, tkg),
+                    tv=names(tv, tvg), dgain_l=self.dgain_l, dgain_g=self.dgain_g, dx=self.dx, dw_g=self.dw_g,
                     dgate_p=self.dgate)
