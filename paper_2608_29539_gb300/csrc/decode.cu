@@ -324,8 +324,14 @@ int launch_decode(DecParams& prm, cudaStream_t st)
         if (set_smem_limit(decode_attn_kernel<D, RING>, DecCfg<D>::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
         attr_done = true;
     }
+    // as many resident CTAs as fit (each keeps one item's K/V load in flight)
+    static int per_sm = 0;
+    if (per_sm == 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_attn_kernel<D, RING>, kDecRows,
+                                                                      DecCfg<D>::kSmemBytes) != cudaSuccess ||
+                        per_sm < 1))
+        per_sm = 2;
     const long long items = static_cast<long long>(prm.B) * prm.Hkv * prm.nchunk;
-    const int grid = static_cast<int>(std::max(1ll, std::min(items, 2ll * device_sm_count())));
+    const int grid = static_cast<int>(std::max(1ll, std::min(items, static_cast<long long>(per_sm) * device_sm_count())));
     decode_attn_kernel<D, RING><<<grid, kDecRows, DecCfg<D>::kSmemBytes, st>>>(prm);
     decode_merge_kernel<D, RING><<<dim3(prm.B, prm.Hq), D, 0, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
