@@ -8,13 +8,15 @@
 //
 // LP is a contraction of 2 d^2 FLOP per row and head against 4 d bytes moved:
 // at d = 128 that is 64 FLOP/byte, more than the CUDA cores can keep up with
-// at HBM speed, so it runs on the tensor cores (warp-level mma.sync over
-// 64-row tiles; per-head operand too small for a tcgen05 tile pipeline to
-// pay).  A block keeps one head's A_h in shared memory and walks a strided
-// share of the row tiles.  The backward computes dU^L = dU^G A_h^T on the same
-// tiles and accumulates dA_h = U^L^T dU^G in registers; per-block partial dA
-// are reduced in block order by a second kernel (deterministic).  SO is
-// elementwise; its ds, db are reduced the same way.
+// at HBM speed, so it runs on the tensor cores.  On every row (K, V) a tcgen05
+// pipeline: TMA brings 128-row tiles of one head into shared memory next to
+// that head's A_h, one thread issues the MMAs into two TMEM buffers, four warps
+// drain them.  On the packed selected rows (Q; rows gathered by position)
+// warp-level mma.sync over 64-row tiles.  A block keeps one head's A_h and
+// walks a strided share of its row tiles.  The backward computes
+// dU^L = dU^G A_h^T on the same tiles and accumulates dA_h = U^L^T dU^G; per-
+// block partial dA are reduced in block order by a second kernel
+// (deterministic).  SO is elementwise; its ds, db are reduced the same way.
 #include <cuda_bf16.h>
 
 #include <cstdint>
@@ -345,6 +347,181 @@ __global__ void __launch_bounds__(256) so_reduce_kernel(const float* __restrict_
     if (dst) dst[x] = s;
 }
 
+// ------------------------------------------------------------------------
+// LP on every row (K and V) with tcgen05: a tile is 128 rows of one head.
+// Roles: warp 0 TMA (A_h once, U tiles through a 2-deep ring), warp 1 MMA
+// issuer (D[128 x D] = U_tile A_h into one of two TMEM buffers), warps 2..5
+// epilogue (TMEM -> bf16 -> global).  A CTA keeps one head; the row tiles of
+// that head are strided over gridDim.x CTAs.  Shared memory: A_h as 64-column
+// halves of [D rows][64] (128-byte swizzle), read as the MN-major B operand;
+// U tiles as 64-column halves of [128 rows][64], the K-major A operand.
+struct LpTcParams {
+    CUtensorMap tm_u;   // u_l [B,T,H,D] as (d, h, t, b), box {64, 1, 128, 1}
+    CUtensorMap tm_a;   // a [H*D rows][D] as (j, 1, row, 1), box {64, 1, D, 1}
+    logo_bf16* u_g;
+    int B, T, H;
+};
+
+template <int D>
+struct LpTcCfg {
+    static constexpr int kHalfA = D * 128;                 // [D rows][64] bf16
+    static constexpr int kABytes = (D / 64) * kHalfA;
+    static constexpr int kHalfU = 128 * 128;               // [128 rows][64] bf16
+    static constexpr int kUBytes = (D / 64) * kHalfU;
+    static constexpr int kOffA = 0;
+    static constexpr int kOffU = kABytes;                  // 2 stages
+    static constexpr int kSmemBytes = kOffU + 2 * kUBytes + 1024;
+    static constexpr uint32_t kTmemCols = D == 128 ? 256 : 128;  // two D-column result buffers
+};
+
+template <int D>
+__global__ void __launch_bounds__(192, 1) lp_tc_fwd_kernel(const __grid_constant__ LpTcParams p)
+{
+    using C = LpTcCfg<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t bar_a, bar_u_full[2], bar_u_empty[2], bar_t_full[2], bar_t_empty[2], bar_drain;
+    __shared__ uint32_t tmem_sh;
+    __shared__ volatile int abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.y;
+    const int tiles_per_seq = (p.T + 127) / 128;
+    const int ntiles = p.B * tiles_per_seq;
+    const uint32_t sA = smem_u32(smem + C::kOffA), sU = smem_u32(smem + C::kOffU);
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        mbar_init(smem_u32(&bar_a), 1);
+        mbar_init(smem_u32(&bar_drain), 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(smem_u32(&bar_u_full[s]), 1);
+            mbar_init(smem_u32(&bar_u_empty[s]), 1);
+            mbar_init(smem_u32(&bar_t_full[s]), 1);
+            mbar_init(smem_u32(&bar_t_empty[s]), 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(&tmem_sh), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_desc(&p.tm_u);
+            tma_prefetch_desc(&p.tm_a);
+            const uint64_t pol_u = policy_evict_first(), pol_a = policy_evict_last();
+            mbar_arrive_expect_tx(smem_u32(&bar_a), C::kABytes);
+            for (int s = 0; s < D / 64; ++s)
+                tma_load_4d(sA + s * C::kHalfA, &p.tm_a, smem_u32(&bar_a), 64 * s, 0, h * D, 0, pol_a);
+            int k = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++k) {
+                const int st = k & 1;
+                if (!(ok = mbar_wait(smem_u32(&bar_u_empty[st]), ((k >> 1) & 1) ^ 1, &abort_flag))) break;
+                const int b = tile / tiles_per_seq, t0 = (tile % tiles_per_seq) * 128;
+                mbar_arrive_expect_tx(smem_u32(&bar_u_full[st]), C::kUBytes);
+                for (int s = 0; s < D / 64; ++s)
+                    tma_load_4d(sU + st * C::kUBytes + s * C::kHalfU, &p.tm_u, smem_u32(&bar_u_full[st]), 64 * s, h,
+                                t0, b, pol_u);
+            }
+            if (!ok) {  // let the copies already issued land before the CTA exits
+                mbar_wait_drain(smem_u32(&bar_a), 0);
+                for (int j = k - 2 > 0 ? k - 2 : 0; j < k; ++j)
+                    mbar_wait_drain(smem_u32(&bar_u_full[j & 1]), (j >> 1) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_bf16_f32(128, D, false, true);
+            bool ok = mbar_wait(smem_u32(&bar_a), 0, &abort_flag);
+            int k = 0;
+            for (int tile = blockIdx.x; ok && tile < ntiles; tile += gridDim.x, ++k) {
+                const int st = k & 1;
+                if (!(ok = mbar_wait(smem_u32(&bar_u_full[st]), (k >> 1) & 1, &abort_flag))) break;
+                if (!(ok = mbar_wait(smem_u32(&bar_t_empty[st]), ((k >> 1) & 1) ^ 1, &abort_flag))) break;
+                tc_fence_after();
+                const uint32_t ub = sU + st * C::kUBytes;
+#pragma unroll
+                for (int ks = 0; ks < D / 16; ++ks) {
+                    const uint32_t ka = (ks >> 2) * C::kHalfU + (ks & 3) * 32;  // U: K-major halves of 64
+                    umma_bf16_ss(tmem + st * D, sdesc_sw128(ub + ka, 16, 1024),
+                                 sdesc_sw128(sA + ks * 2048, C::kHalfA, 1024), idesc, ks > 0 ? 1u : 0u);
+                }
+                umma_commit(smem_u32(&bar_u_empty[st]));
+                umma_commit(smem_u32(&bar_t_full[st]));
+            }
+            if (!ok) {
+                umma_commit(smem_u32(&bar_drain));
+                mbar_wait_drain(smem_u32(&bar_drain), 0);
+            }
+        }
+    } else {
+        // epilogue: warp w reads TMEM lanes 32 (w % 4) .. (its rows of the tile)
+        const int quad = warp & 3;
+        const int r = quad * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        int k = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++k) {
+            const int st = k & 1;
+            const bool ok = mbar_wait(smem_u32(&bar_t_full[st]), (k >> 1) & 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            tc_fence_after();
+            const int b = tile / tiles_per_seq, t = (tile % tiles_per_seq) * 128 + r;
+            logo_bf16* dst = p.u_g + ((static_cast<int64_t>(b) * p.T + t) * p.H + h) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem + lane_off + st * D + c * 32, v);
+                tmem_wait_ld();
+                if (c == D / 32 - 1) {
+                    tc_fence_before();
+                    mbar_arrive(smem_u32(&bar_t_empty[st]));
+                }
+                if (t < p.T) {
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(v[8 * q4 + 0]), __uint_as_float(v[8 * q4 + 1]));
+                        w.y = pack_bf16x2(__uint_as_float(v[8 * q4 + 2]), __uint_as_float(v[8 * q4 + 3]));
+                        w.z = pack_bf16x2(__uint_as_float(v[8 * q4 + 4]), __uint_as_float(v[8 * q4 + 5]));
+                        w.w = pack_bf16x2(__uint_as_float(v[8 * q4 + 6]), __uint_as_float(v[8 * q4 + 7]));
+                        *reinterpret_cast<uint4*>(dst + c * 32 + q4 * 8) = w;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+template <int D>
+int launch_lp_tc_fwd(const logo_bf16* u_l, const logo_bf16* a, const logo_dims& d, logo_bf16* u_g, cudaStream_t st)
+{
+    LpTcParams prm{};
+    if (!encode_bf16_4d(&prm.tm_u, u_l, D, d.Hq, d.T, d.B, 64, 128) ||
+        !encode_bf16_4d(&prm.tm_a, a, D, 1, static_cast<uint64_t>(d.Hq) * D, 1, 64, D))
+        return LOGO_ERR_CUDA;
+    prm.u_g = u_g;
+    prm.B = d.B;
+    prm.T = d.T;
+    prm.H = d.Hq;
+    if (set_smem_limit(lp_tc_fwd_kernel<D>, LpTcCfg<D>::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+    const int ntiles = d.B * ((d.T + 127) / 128);
+    int per_head = (2 * device_sm_count()) / d.Hq;
+    per_head = per_head < 1 ? 1 : (per_head > ntiles ? ntiles : per_head);
+    lp_tc_fwd_kernel<D><<<dim3(per_head, d.Hq), 192, LpTcCfg<D>::kSmemBytes, st>>>(prm);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
 int so_vpt(const logo_dims& d)
 {
     const int nvec = d.Hq * d.D / 8;
@@ -411,7 +588,11 @@ extern "C" int logo_branch_transform(const logo_bf16* u_l, const logo_bf16* a_lp
     if (a_lp && !aligned16(a_lp)) return LOGO_ERR_UNSUPPORTED;
     const RowSet R{pos, cu_q, n_sel_total, dims.B, dims.T};
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (a_lp) {
+    if (a_lp && !pos) {  // every row: the tcgen05 pipeline
+        return dims.D == 128 ? launch_lp_tc_fwd<128>(u_l, a_lp, dims, u_g, st)
+                             : launch_lp_tc_fwd<64>(u_l, a_lp, dims, u_g, st);
+    }
+    if (a_lp) {  // the packed selected rows (Q): warp-level MMA over gathered rows
         return dims.D == 128 ? launch_lp_fwd<128>(u_l, a_lp, R, dims.Hq, u_g, st)
                              : launch_lp_fwd<64>(u_l, a_lp, R, dims.Hq, u_g, st);
     }
