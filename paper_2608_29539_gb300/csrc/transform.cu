@@ -522,6 +522,232 @@ int launch_lp_tc_fwd(const logo_bf16* u_l, const logo_bf16* a, const logo_dims& 
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
+// LP backward on every row, d = 128, with tcgen05.  Per 128-row tile of one
+// head: dU = dG A_h^T (A_h read as the K-major B operand: its rows are the
+// output dimension i, its columns the contracted j) into one of two TMEM
+// buffers, drained to du_l by warps 2..5; and dA_h += U^T dG (both tiles read
+// as MN-major operands: rows are the contracted dimension) accumulated in TMEM
+// over all the CTA's tiles, written as the CTA's partial at the end.
+struct LpTcBwdParams {
+    CUtensorMap tm_u, tm_g, tm_a;
+    logo_bf16* du_l;
+    float* part;  // [H][gridDim.x][D][D]
+    int B, T, H, accumulate;
+};
+
+struct LpTcBwdCfg {
+    static constexpr int D = 128;
+    static constexpr int kHalf = 128 * 128;          // [128 rows][64] bf16
+    static constexpr int kTile = 2 * kHalf;          // 128 rows x 128
+    static constexpr int kOffA = 0;
+    static constexpr int kOffU = kTile;              // 2 stages of (U, G)
+    static constexpr int kSmemBytes = kOffU + 4 * kTile + 1024;
+    static constexpr uint32_t kColDA = 256;          // dU buffers at 0 and 128
+    static constexpr uint32_t kTmemCols = 512;
+};
+
+__global__ void __launch_bounds__(192, 1) lp_tc_bwd_kernel(const __grid_constant__ LpTcBwdParams p)
+{
+    using C = LpTcBwdCfg;
+    constexpr int D = C::D;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t bar_a, bar_in_full[2], bar_in_empty[2], bar_t_full[2], bar_t_empty[2];
+    __shared__ __align__(8) uint64_t bar_da, bar_drain;
+    __shared__ uint32_t tmem_sh;
+    __shared__ volatile int abort_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.y;
+    const int tiles_per_seq = (p.T + 127) / 128;
+    const int ntiles = p.B * tiles_per_seq;
+    const uint32_t sA = smem_u32(smem + C::kOffA), sIn = smem_u32(smem + C::kOffU);
+    if (threadIdx.x == 0) {
+        abort_flag = 0;
+        mbar_init(smem_u32(&bar_a), 1);
+        mbar_init(smem_u32(&bar_da), 1);
+        mbar_init(smem_u32(&bar_drain), 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(smem_u32(&bar_in_full[s]), 1);
+            mbar_init(smem_u32(&bar_in_empty[s]), 1);
+            mbar_init(smem_u32(&bar_t_full[s]), 1);
+            mbar_init(smem_u32(&bar_t_empty[s]), 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(&tmem_sh), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch_desc(&p.tm_u);
+            tma_prefetch_desc(&p.tm_g);
+            tma_prefetch_desc(&p.tm_a);
+            const uint64_t pol = policy_evict_first(), pol_a = policy_evict_last();
+            mbar_arrive_expect_tx(smem_u32(&bar_a), C::kTile);
+            for (int s = 0; s < 2; ++s) tma_load_4d(sA + s * C::kHalf, &p.tm_a, smem_u32(&bar_a), 64 * s, 0, h * D, 0, pol_a);
+            int k = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++k) {
+                const int st = k & 1;
+                if (!(ok = mbar_wait(smem_u32(&bar_in_empty[st]), ((k >> 1) & 1) ^ 1, &abort_flag))) break;
+                const int b = tile / tiles_per_seq, t0 = (tile % tiles_per_seq) * 128;
+                const uint32_t bar = smem_u32(&bar_in_full[st]);
+                const uint32_t ub = sIn + st * 2 * C::kTile, gb = ub + C::kTile;
+                mbar_arrive_expect_tx(bar, 2 * C::kTile);
+                for (int s = 0; s < 2; ++s) {
+                    tma_load_4d(ub + s * C::kHalf, &p.tm_u, bar, 64 * s, h, t0, b, pol);
+                    tma_load_4d(gb + s * C::kHalf, &p.tm_g, bar, 64 * s, h, t0, b, pol);
+                }
+            }
+            if (!ok) {
+                mbar_wait_drain(smem_u32(&bar_a), 0);
+                for (int j = k - 2 > 0 ? k - 2 : 0; j < k; ++j)
+                    mbar_wait_drain(smem_u32(&bar_in_full[j & 1]), (j >> 1) & 1);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t id_du = idesc_bf16_f32(128, D, false, false);  // G K-major x A_h K-major
+            constexpr uint32_t id_da = idesc_bf16_f32(D, D, true, true);      // U^T, G: both MN-major
+            bool ok = mbar_wait(smem_u32(&bar_a), 0, &abort_flag);
+            int k = 0;
+            for (int tile = blockIdx.x; ok && tile < ntiles; tile += gridDim.x, ++k) {
+                const int st = k & 1;
+                if (!(ok = mbar_wait(smem_u32(&bar_in_full[st]), (k >> 1) & 1, &abort_flag))) break;
+                if (!(ok = mbar_wait(smem_u32(&bar_t_empty[st]), ((k >> 1) & 1) ^ 1, &abort_flag))) break;
+                tc_fence_after();
+                const uint32_t ub = sIn + st * 2 * C::kTile, gb = ub + C::kTile;
+#pragma unroll
+                for (int ks = 0; ks < D / 16; ++ks) {  // contracted: j
+                    const uint32_t off = (ks >> 2) * C::kHalf + (ks & 3) * 32;
+                    umma_bf16_ss(tmem + st * D, sdesc_sw128(gb + off, 16, 1024), sdesc_sw128(sA + off, 16, 1024), id_du,
+                                 ks > 0 ? 1u : 0u);
+                }
+#pragma unroll
+                for (int ks = 0; ks < 128 / 16; ++ks) {  // contracted: the tile's rows
+                    umma_bf16_ss(tmem + C::kColDA, sdesc_sw128(ub + ks * 2048, C::kHalf, 1024),
+                                 sdesc_sw128(gb + ks * 2048, C::kHalf, 1024), id_da, (k > 0 || ks > 0) ? 1u : 0u);
+                }
+                umma_commit(smem_u32(&bar_in_empty[st]));
+                umma_commit(smem_u32(&bar_t_full[st]));
+            }
+            // dA complete (every MMA of this thread before the commit); also on a
+            // CTA with no tile, so that the epilogue's final wait ends
+            if (ok) umma_commit(smem_u32(&bar_da));
+            if (!ok) {
+                umma_commit(smem_u32(&bar_drain));
+                mbar_wait_drain(smem_u32(&bar_drain), 0);
+            }
+        }
+    } else {
+        const int quad = warp & 3;
+        const int r = quad * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        int k = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++k) {
+            const int st = k & 1;
+            ok = mbar_wait(smem_u32(&bar_t_full[st]), (k >> 1) & 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            tc_fence_after();
+            const int b = tile / tiles_per_seq, t = (tile % tiles_per_seq) * 128 + r;
+            logo_bf16* dst = p.du_l + ((static_cast<int64_t>(b) * p.T + t) * p.H + h) * D;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem + lane_off + st * D + c * 32, v);
+                tmem_wait_ld();
+                if (c == D / 32 - 1) {
+                    tc_fence_before();
+                    mbar_arrive(smem_u32(&bar_t_empty[st]));
+                }
+                if (t < p.T) {
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        float x[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) x[e] = __uint_as_float(v[8 * q4 + e]);
+                        uint4* dp = reinterpret_cast<uint4*>(dst + c * 32 + q4 * 8);
+                        if (p.accumulate) {
+                            const uint4 old = *dp;
+                            const __nv_bfloat162* o2 = reinterpret_cast<const __nv_bfloat162*>(&old);
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float2 f = __bfloat1622float2(o2[e]);
+                                x[2 * e] += f.x;
+                                x[2 * e + 1] += f.y;
+                            }
+                        }
+                        uint4 w;
+                        w.x = pack_bf16x2(x[0], x[1]);
+                        w.y = pack_bf16x2(x[2], x[3]);
+                        w.z = pack_bf16x2(x[4], x[5]);
+                        w.w = pack_bf16x2(x[6], x[7]);
+                        *dp = w;
+                    }
+                }
+            }
+        }
+        // the CTA's dA partial: lane r holds row i = r, columns j
+        float* pp = p.part + ((static_cast<int64_t>(h) * gridDim.x + blockIdx.x) * D + r) * D;
+        if (ok && k == 0) {  // no tile: a zero partial (the launch gives every CTA one)
+            for (int j = 0; j < D; j += 4) *reinterpret_cast<float4*>(pp + j) = make_float4(0.f, 0.f, 0.f, 0.f);
+        } else if (ok && mbar_wait(smem_u32(&bar_da), 0, &abort_flag)) {
+            tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem + lane_off + C::kColDA + c * 32, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int e = 0; e < 32; e += 4)
+                    *reinterpret_cast<float4*>(pp + c * 32 + e) =
+                        make_float4(__uint_as_float(v[e]), __uint_as_float(v[e + 1]), __uint_as_float(v[e + 2]),
+                                    __uint_as_float(v[e + 3]));
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+int launch_lp_tc_bwd(const logo_bf16* u_l, const logo_bf16* a, const logo_bf16* du_g, const logo_dims& d,
+                     logo_bf16* du_l, int accumulate, float* da, float* part, cudaStream_t st)
+{
+    constexpr int D = 128;
+    LpTcBwdParams prm{};
+    if (!encode_bf16_4d(&prm.tm_u, u_l, D, d.Hq, d.T, d.B, 64, 128) ||
+        !encode_bf16_4d(&prm.tm_g, du_g, D, d.Hq, d.T, d.B, 64, 128) ||
+        !encode_bf16_4d(&prm.tm_a, a, D, 1, static_cast<uint64_t>(d.Hq) * D, 1, 64, D))
+        return LOGO_ERR_CUDA;
+    prm.du_l = du_l;
+    prm.part = part;
+    prm.B = d.B;
+    prm.T = d.T;
+    prm.H = d.Hq;
+    prm.accumulate = accumulate;
+    if (set_smem_limit(lp_tc_bwd_kernel, LpTcBwdCfg::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+    const int ntiles = d.B * ((d.T + 127) / 128);
+    int per_head = device_sm_count() / d.Hq;
+    per_head = per_head < 1 ? 1 : (per_head > ntiles ? ntiles : per_head);
+    per_head = per_head > kChunksPerHead ? kChunksPerHead : per_head;  // the workspace holds that many partials
+    lp_tc_bwd_kernel<<<dim3(per_head, d.Hq), 192, LpTcBwdCfg::kSmemBytes, st>>>(prm);
+    if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
+    const int64_t total = static_cast<int64_t>(d.Hq) * D * D;
+    reduce_parts_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(part, per_head, D * D, d.Hq, da);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+}
+
 int so_vpt(const logo_dims& d)
 {
     const int nvec = d.Hq * d.D / 8;
@@ -631,6 +857,8 @@ extern "C" int logo_branch_transform_bwd(const logo_bf16* u_l, const logo_bf16* 
     const RowSet R{pos, cu_q, n_sel_total, dims.B, dims.T};
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     float* part = static_cast<float*>(workspace);
+    if (a_lp && !pos && dims.D == 128)  // every row: the tcgen05 pipeline
+        return launch_lp_tc_bwd(u_l, a_lp, du_g, dims, du_l, accumulate, da_lp, part, st);
     if (a_lp) {
         return dims.D == 128 ? launch_lp_bwd<128>(u_l, a_lp, du_g, R, dims.Hq, du_l, accumulate, da_lp, part, st)
                              : launch_lp_bwd<64>(u_l, a_lp, du_g, R, dims.Hq, du_l, accumulate, da_lp, part, st);
