@@ -671,13 +671,15 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                         umma_bf16_ss(tmem + C::kColDK, sdesc_sw128(db + ks * 32, 16, 1024),
                                      sdesc_sw128(qb + ks * 2048, 8192, 1024), idKV, acc);
                     }
+                    // Q, dO of tile u are read: release the ring stage before dQ^T
+                    // (which reads K and dS^T only), so the next load starts earlier
+                    umma_commit(smem_u32(&bar_qdo_empty[st]));
 #pragma unroll
                     for (int ks = 0; ks < kBN / 16; ++ks) {
                         umma_bf16_ss(tmem + C::kColDQ, sdesc_sw128(sK + ks * 2048, 16384, 1024),
                                      sdesc_sw128(db + ks * 2048, 16384, 1024), idQ, ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_dq_full[b]));
-                    umma_commit(smem_u32(&bar_qdo_empty[st]));
                 }
                 if (!ok) break;
                 // the item's last reads of K and V (S^T, dP^T of issuer A finished before ds_full)
@@ -756,11 +758,6 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 ok = mbar_wait(smem_u32(&bar_st_full), u & 1, &abort_flag);
                 __syncwarp();
                 if (!ok) break;
-                // P^T (TMEM) / dS^T (shared) buffer b is free once the MMAs of tile u-2 are done
-                // (they were issued before S^T of tile u, so this rarely waits)
-                ok = mbar_wait(smem_u32(&bar_dq_full[b]), ((u >> 1) & 1) ^ 1, &abort_flag);
-                __syncwarp();
-                if (!ok) break;
                 tc_fence_after();
                 uint32_t sv[32], dpv[32];
                 tmem_ld32(tmem + lane_off + C::kColS + half * 32, sv);
@@ -799,6 +796,13 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                 };
                 if (open) columns(std::false_type{});
                 else columns(std::true_type{});
+                // P^T (TMEM) / dS^T (shared) buffer b is free once the MMAs of tile
+                // u-2 are done.  Waiting here rather than before the loads lets
+                // S^T, dP^T of tile u+1 enter the MMA queue earlier.
+                ok = mbar_wait(smem_u32(&bar_dq_full[b]), ((u >> 1) & 1) ^ 1, &abort_flag);
+                __syncwarp();
+                if (!ok) break;
+                tc_fence_after();
                 // P^T row t: query columns half*32.. as 16 bf16 pairs, the TMEM
                 // operand layout (column c holds queries 2c, 2c+1)
                 tmem_st16(tmem + lane_off + C::kColP + 32 * b + half * 16, pk);
