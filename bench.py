@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "a9e31f5a2c17cf68"): 823936000 + 479489280,
-    ("global_bwd", "a9e31f5a2c17cf68"): 471555840 + 433355008,
+    ("local_bwd", "09669b4ffbb09292"): 826112512 + 479320832,
+    ("global_bwd", "09669b4ffbb09292"): 470733568 + 431303936,
 }
 
 
