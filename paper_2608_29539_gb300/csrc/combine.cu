@@ -9,12 +9,13 @@
 // flight), and the D/8 lanes of a head reduce their sums with warp shuffles.
 // The backward sums dp_t over every head of the token in shared memory, and
 // the gain gradients over tokens in registers (fixed vectors per thread), then
-// per block into a workspace that a second kernel reduces in block order
-// (deterministic).  All arithmetic is fp32; inputs and outputs bf16.
+// per block into a workspace that a second kernel sums in a fixed order
+// (colsum.cuh: deterministic).  All arithmetic is fp32; inputs and outputs bf16.
 #include <cuda_bf16.h>
 
 #include <cstdint>
 
+#include "colsum.cuh"
 #include "host_common.h"
 #include "logo_status.cuh"
 
@@ -257,20 +258,6 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     }
 }
 
-// dgain_{l,g}[e] = sum over blocks b (in order) of part[b][{0,1}][e].
-__global__ void __launch_bounds__(256) combine_dgain_reduce_kernel(const float* __restrict__ part, int nblk, int hd,
-                                                                   float* __restrict__ dgain_l,
-                                                                   float* __restrict__ dgain_g)
-{
-    const int e = blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= 2 * hd) return;
-    const int w = e / hd, x = e % hd;
-    float s = 0.f;
-    for (int b = 0; b < nblk; ++b) s += part[(static_cast<int64_t>(b) * 2 + w) * hd + x];
-    float* dst = w == 0 ? dgain_l : dgain_g;
-    if (dst) dst[x] = s;
-}
-
 int vec_per_thread(const logo_dims& d)
 {
     const int nvec = d.Hq * (d.D / 8);
@@ -389,8 +376,8 @@ int combine_bwd_common(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf1
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     if (gains) {
         const int hd = dims.Hq * dims.D;
-        combine_dgain_reduce_kernel<<<(2 * hd + 255) / 256, 256, 0, st>>>(part, static_cast<int>(grid), hd, dgain_l,
-                                                                          dgain_g);
+        colsum_kernel<<<colsum_blocks(2 * hd), kColSumThreads, 0, st>>>(part, static_cast<int>(grid), 2 * hd, hd,
+                                                                        dgain_l, dgain_g);
         if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     }
     return LOGO_OK;

@@ -9,11 +9,13 @@
 // dw_g = sum_t dlogit_t x_t with dlogit_t = dp_t p_t (1 - p_t): a thread owns
 // fixed 8-wide slices of d_model for all the tokens of its block (two tokens
 // per step, so the loads of both are in flight together), and the per-block
-// sums are reduced in block order by a second kernel (deterministic).
+// sums are added by a second kernel in a fixed order (colsum.cuh:
+// deterministic).
 #include <cuda_bf16.h>
 
 #include <cstdint>
 
+#include "colsum.cuh"
 #include "host_common.h"
 
 namespace logo {
@@ -148,17 +150,6 @@ __global__ void __launch_bounds__(kBwdThreads) gate_bwd_kernel(const logo_bf16* 
     }
 }
 
-// dw[i] = sum over blocks b (in order) of part[b][i].
-__global__ void __launch_bounds__(256) gate_dw_reduce_kernel(const float* __restrict__ part, int nblk, int dm,
-                                                             float* __restrict__ dw)
-{
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= dm) return;
-    float s = 0.f;
-    for (int b = 0; b < nblk; ++b) s += part[static_cast<int64_t>(b) * dm + i];
-    dw[i] = s;
-}
-
 int gate_vpt(int dm)
 {
     const int nv = dm / 8;
@@ -248,7 +239,8 @@ extern "C" int logo_gate_bwd(const logo_bf16* x, const float* w_g, const float* 
     }
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     if (dw_g) {
-        gate_dw_reduce_kernel<<<(d_model + 255) / 256, 256, 0, st>>>(part, static_cast<int>(grid), d_model, dw_g);
+        colsum_kernel<<<colsum_blocks(d_model), kColSumThreads, 0, st>>>(part, static_cast<int>(grid), d_model, d_model,
+                                                                         dw_g, nullptr);
         if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     }
     return LOGO_OK;

@@ -16,11 +16,13 @@
 // walks a strided share of its row tiles.  The backward computes
 // dU^L = dU^G A_h^T on the same tiles and accumulates dA_h = U^L^T dU^G; per-
 // block partial dA are reduced in block order by a second kernel
-// (deterministic).  SO is elementwise; its ds, db are reduced the same way.
+// (deterministic).  SO is elementwise; its per-block ds, db are summed by the
+// fixed-order column sum of colsum.cuh (deterministic too).
 #include <cuda_bf16.h>
 
 #include <cstdint>
 
+#include "colsum.cuh"
 #include "attn_common.cuh"
 #include "host_common.h"
 #include "sm100.cuh"
@@ -332,19 +334,6 @@ __global__ void __launch_bounds__(256) so_bwd_kernel(const logo_bf16* __restrict
             part[static_cast<int64_t>(blockIdx.x) * 2 * hd + hd + v * 8 + i] = acc_b[k][i];
         }
     }
-}
-
-// ds / db from the [grid][2][H*D] parts (block order).
-__global__ void __launch_bounds__(256) so_reduce_kernel(const float* __restrict__ part, int nblk, int hd,
-                                                        float* __restrict__ ds, float* __restrict__ db)
-{
-    const int e = blockIdx.x * blockDim.x + threadIdx.x;
-    if (e >= 2 * hd) return;
-    const int w = e / hd, x = e % hd;
-    float s = 0.f;
-    for (int b = 0; b < nblk; ++b) s += part[(static_cast<int64_t>(b) * 2 + w) * hd + x];
-    float* dst = w == 0 ? ds : db;
-    if (dst) dst[x] = s;
 }
 
 // ------------------------------------------------------------------------
@@ -871,6 +860,6 @@ extern "C" int logo_branch_transform_bwd(const logo_bf16* u_l, const logo_bf16* 
     }
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     const int hd = dims.Hq * dims.D;
-    so_reduce_kernel<<<(2 * hd + 255) / 256, 256, 0, st>>>(part, grid, hd, ds_so, db_so);
+    colsum_kernel<<<colsum_blocks(2 * hd), kColSumThreads, 0, st>>>(part, grid, 2 * hd, hd, ds_so, db_so);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
