@@ -275,10 +275,22 @@ __global__ void __launch_bounds__(kDecRows, 2) decode_attn_kernel(const __grid_c
 
 // Exact combination of the chunks of one (row, head):
 // M = max m_c, L = sum l_c 2^(m_c - M), o = sum o_c 2^(m_c - M) / L.
+// kMergeSplit x D threads per (row, head): a block max of the chunk maxima,
+// then in batches of the block's size the chunk weights go to shared memory
+// and thread (q, d) adds o_c[d] w_c over the chunks c = q (mod kMergeSplit);
+// the partial sums are added in a fixed order (deterministic).  One thread
+// per d walking every chunk twice left this step bound by load latency.
+constexpr int kMergeSplit = 4;
+
 template <int D, bool RING>
-__global__ void __launch_bounds__(D) decode_merge_kernel(const __grid_constant__ DecParams p)
+__global__ void __launch_bounds__(kMergeSplit * D) decode_merge_kernel(const __grid_constant__ DecParams p)
 {
-    const int r = blockIdx.x, h = blockIdx.y, d = threadIdx.x;
+    constexpr int NT = kMergeSplit * D;
+    __shared__ float sh_w[NT];
+    __shared__ float sh_red[NT / 32];
+    __shared__ float sh_o[kMergeSplit][D];
+    const int r = blockIdx.x, h = blockIdx.y, t = threadIdx.x;
+    const int d = t % D, q = t / D;
     int b = r;
     if (!RING) {
         if (r >= *p.n_sel) return;
@@ -287,19 +299,47 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const __grid_constant__
     const int len = RING ? p.seq_len[b] : min(p.seq_len[b], p.R);
     const int nc = (min(max(len, 0), p.R) + kDecRows - 1) / kDecRows;
     const float* base = p.part + (static_cast<int64_t>(r) * p.Hq + h) * p.nchunk * (D + 2);
+    // M: strided over the threads, then warps, then the block
     float M = -INFINITY;
-    for (int c = 0; c < nc; ++c) M = fmaxf(M, base[c * (D + 2) + D]);
+    for (int c = t; c < nc; c += NT) M = fmaxf(M, base[c * (D + 2) + D]);
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    if ((t & 31) == 0) sh_red[t >> 5] = M;
+    __syncthreads();
+    M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < NT / 32; ++w) M = fmaxf(M, sh_red[w]);
     const float M_use = M == -INFINITY ? 0.f : M;
     float L = 0.f, o = 0.f;
-    for (int c = 0; c < nc; ++c) {
-        const float* pc = base + c * (D + 2);
-        const float w = ex2_approx(pc[D] - M_use);
-        L += pc[D + 1] * w;
-        o += pc[d] * w;
+    for (int c0 = 0; c0 < nc; c0 += NT) {
+        __syncthreads();  // the previous batch's weights are consumed
+        if (c0 + t < nc) {
+            const float* pc = base + (c0 + t) * (D + 2);
+            const float w = ex2_approx(pc[D] - M_use);
+            sh_w[t] = w;
+            L += pc[D + 1] * w;
+        }
+        __syncthreads();
+        const int nb = min(NT, nc - c0);
+#pragma unroll 4
+        for (int k = q; k < nb; k += kMergeSplit) o += base[(c0 + k) * (D + 2) + d] * sh_w[k];
     }
-    const float val = L > 0.f ? o / L : 0.f;
-    const __nv_bfloat16 bv = __float2bfloat16_rn(val);
-    p.out[(static_cast<int64_t>(r) * p.Hq + h) * D + d] = *reinterpret_cast<const logo_bf16*>(&bv);
+    // L over the block (warps in order), o over the kMergeSplit lanes of each d
+    for (int s2 = 16; s2 > 0; s2 >>= 1) L += __shfl_xor_sync(0xffffffffu, L, s2);
+    __syncthreads();
+    if ((t & 31) == 0) sh_red[t >> 5] = L;
+    sh_o[q][d] = o;
+    __syncthreads();
+    if (q == 0) {
+        float Lt = 0.f;
+#pragma unroll
+        for (int w = 0; w < NT / 32; ++w) Lt += sh_red[w];
+        float ot = 0.f;
+#pragma unroll
+        for (int k = 0; k < kMergeSplit; ++k) ot += sh_o[k][d];
+        const float val = Lt > 0.f ? ot / Lt : 0.f;
+        const __nv_bfloat16 bv = __float2bfloat16_rn(val);
+        p.out[(static_cast<int64_t>(r) * p.Hq + h) * D + d] = *reinterpret_cast<const logo_bf16*>(&bv);
+    }
 }
 
 size_t decode_ws_bytes(const logo_dims& d)
@@ -333,7 +373,7 @@ int launch_decode(DecParams& prm, cudaStream_t st)
     const long long items = static_cast<long long>(prm.B) * prm.Hkv * prm.nchunk;
     const int grid = static_cast<int>(std::max(1ll, std::min(items, static_cast<long long>(per_sm) * device_sm_count())));
     decode_attn_kernel<D, RING><<<grid, kDecRows, DecCfg<D>::kSmemBytes, st>>>(prm);
-    decode_merge_kernel<D, RING><<<dim3(prm.B, prm.Hq), D, 0, st>>>(prm);
+    decode_merge_kernel<D, RING><<<dim3(prm.B, prm.Hq), kMergeSplit * D, 0, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
