@@ -11,13 +11,18 @@
 // the gain gradients over tokens in registers (fixed vectors per thread), then
 // per block into a workspace that a second kernel sums in a fixed order
 // (colsum.cuh: deterministic).  All arithmetic is fp32; inputs and outputs bf16.
+// The kernels are bound as much by instruction issue as by HBM: without gains
+// (both NULL, i.e. 1) a separate instantiation drops the gain loads and the
+// unit multiplies and does the elementwise work as f32x2 pairs.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cstdint>
 
 #include "colsum.cuh"
 #include "host_common.h"
 #include "logo_status.cuh"
+#include "sm100.cuh"
 
 namespace logo {
 namespace {
@@ -69,6 +74,43 @@ __device__ __forceinline__ Vec8 load_gain(const float* g, int h, int D, int j)
     return r;
 }
 
+// sum_i x_i^2 and sum_i x_i y_i over a vector of 8, as f32x2 pairs
+__device__ __forceinline__ float sumsq8(const Vec8& x)
+{
+    uint64_t a = f2_mul(f2_pack(x.v[0], x.v[1]), f2_pack(x.v[0], x.v[1]));
+    uint64_t b = f2_mul(f2_pack(x.v[2], x.v[3]), f2_pack(x.v[2], x.v[3]));
+    a = f2_fma(f2_pack(x.v[4], x.v[5]), f2_pack(x.v[4], x.v[5]), a);
+    b = f2_fma(f2_pack(x.v[6], x.v[7]), f2_pack(x.v[6], x.v[7]), b);
+    float lo, hi;
+    f2_unpack(f2_add(a, b), lo, hi);
+    return lo + hi;
+}
+
+__device__ __forceinline__ float dot8(const Vec8& x, const Vec8& y)
+{
+    uint64_t a = f2_mul(f2_pack(x.v[0], x.v[1]), f2_pack(y.v[0], y.v[1]));
+    uint64_t b = f2_mul(f2_pack(x.v[2], x.v[3]), f2_pack(y.v[2], y.v[3]));
+    a = f2_fma(f2_pack(x.v[4], x.v[5]), f2_pack(y.v[4], y.v[5]), a);
+    b = f2_fma(f2_pack(x.v[6], x.v[7]), f2_pack(y.v[6], y.v[7]), b);
+    float lo, hi;
+    f2_unpack(f2_add(a, b), lo, hi);
+    return lo + hi;
+}
+
+// x * a + y * b elementwise (y, b optional), as f32x2 pairs
+__device__ __forceinline__ Vec8 axpby8(const Vec8& x, float a, const Vec8* y, float b)
+{
+    const uint64_t a2 = f2_pack(a, a), b2 = f2_pack(b, b);
+    Vec8 r;
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) {
+        uint64_t t = f2_mul(f2_pack(x.v[i], x.v[i + 1]), a2);
+        if (y) t = f2_fma(f2_pack(y->v[i], y->v[i + 1]), b2, t);
+        f2_unpack(t, r.v[i], r.v[i + 1]);
+    }
+    return r;
+}
+
 // Sum over the `width` consecutive lanes (a power of two <= 32) of one head.
 __device__ __forceinline__ float head_sum(float x, int width)
 {
@@ -76,7 +118,7 @@ __device__ __forceinline__ float head_sum(float x, int width)
     return x;
 }
 
-template <int VPT>
+template <int VPT, bool UNIT>
 __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
     const logo_bf16* __restrict__ o_l, const logo_bf16* __restrict__ o_c, const float* __restrict__ gate_p,
     const uint8_t* __restrict__ z, const int32_t* __restrict__ row_of, const float* __restrict__ gain_l,
@@ -103,16 +145,26 @@ __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
             const bool active = v < nvec;
             const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
             const Vec8 xl = unpack8(rl[k]);
+            Vec8 out;
+            float r_l, r_g = 0.f;
+            if constexpr (UNIT) {
+                r_l = rsqrtf(head_sum(sumsq8(xl), vpr) * inv_d + eps);
+                if (sel) {
+                    const Vec8 xg = unpack8(rg[k]);
+                    r_g = rsqrtf(head_sum(sumsq8(xg), vpr) * inv_d + eps);
+                    out = axpby8(xl, (1.0f - pt) * r_l, &xg, pt * r_g);
+                } else {
+                    out = axpby8(xl, r_l, nullptr, 0.f);
+                }
+            } else {
             float ss = 0.f;
 #pragma unroll
             for (int i = 0; i < 8; ++i) ss += xl.v[i] * xl.v[i];
             ss = head_sum(ss, vpr);
-            const float r_l = rsqrtf(ss * inv_d + eps);
+            r_l = rsqrtf(ss * inv_d + eps);
             const Vec8 gl = load_gain(gain_l, h, D, j);
-            Vec8 out;
 #pragma unroll
             for (int i = 0; i < 8; ++i) out.v[i] = xl.v[i] * r_l * gl.v[i];
-            float r_g = 0.f;
             if (sel) {
                 const Vec8 xg = unpack8(rg[k]);
                 float sg = 0.f;
@@ -123,6 +175,7 @@ __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
                 const Vec8 gg = load_gain(gain_g, h, D, j);
 #pragma unroll
                 for (int i = 0; i < 8; ++i) out.v[i] = (1.0f - pt) * out.v[i] + pt * (xg.v[i] * r_g * gg.v[i]);
+            }
             }
             if (active) {
                 store_bf16x8(o + (bt * nvec + v) * 8, out);
@@ -137,7 +190,7 @@ __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
 
 // part (DGAIN): [gridDim.x][2][H*D] float32 per-block sums of the local and
 // global gain gradients.
-template <int VPT, bool DGAIN>
+template <int VPT, bool DGAIN, bool UNIT>
 __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     const logo_bf16* __restrict__ dO, const logo_bf16* __restrict__ o_l, const logo_bf16* __restrict__ o_c,
     const float* __restrict__ gate_p, const uint8_t* __restrict__ z, const int32_t* __restrict__ row_of,
@@ -171,6 +224,7 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
             rg[k] = (sel && active) ? ld_vec(o_c + (row * nvec + v) * 8) : make_uint4(0, 0, 0, 0);
         }
         float dp_acc = 0.f;
+        uint64_t dp2 = 0ull;  // UNIT: dp as f32x2 pairs
 #pragma unroll
         for (int k = 0; k < VPT; ++k) {
             const int v = threadIdx.x + k * kThreads;
@@ -178,6 +232,39 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
             const int h = active ? v / vpr : 0, j = active ? v % vpr : 0;
             const Vec8 g = unpack8(rd[k]);
             const Vec8 xl = unpack8(rl[k]);
+            if constexpr (UNIT) {
+                // gains 1: dx = r dy - x r^3 mean(x dy), dy = w dO
+                const float ss = head_sum(sumsq8(xl), vpr);
+                const float xgdy = head_sum(dot8(xl, g), vpr) * wl;
+                const float r_l = rsqrtf(ss * inv_d + eps);
+                const float cl = r_l * r_l * r_l * xgdy * inv_d;
+                if (active) store_bf16x8(dO_l + (bt * nvec + v) * 8, axpby8(g, r_l * wl, &xl, -cl));
+                if constexpr (DGAIN) {  // d gain_l = dy * x r
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) accL[k][i] += g.v[i] * wl * xl.v[i] * r_l;
+                }
+                if (sel) {
+                    const Vec8 xg = unpack8(rg[k]);
+                    const float sg = head_sum(sumsq8(xg), vpr);
+                    const float xgdyg = head_sum(dot8(xg, g), vpr) * pt;
+                    const float r_g = rsqrtf(sg * inv_d + eps);
+                    const float cg = r_g * r_g * r_g * xgdyg * inv_d;
+                    if (active) store_bf16x8(dO_c + (row * nvec + v) * 8, axpby8(g, r_g * pt, &xg, -cg));
+                    if constexpr (DGAIN) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) accG[k][i] += g.v[i] * pt * xg.v[i] * r_g;
+                    }
+                    // dp += dO . (xg r_g - xl r_l)
+                    const uint64_t rg2 = f2_pack(r_g, r_g), rl2 = f2_pack(-r_l, -r_l);
+#pragma unroll
+                    for (int i = 0; i < 8; i += 2) {
+                        const uint64_t t = f2_fma(f2_pack(xl.v[i], xl.v[i + 1]), rl2,
+                                                  f2_mul(f2_pack(xg.v[i], xg.v[i + 1]), rg2));
+                        dp2 = f2_fma(f2_pack(g.v[i], g.v[i + 1]), t, dp2);
+                    }
+                }
+                continue;
+            }
             const Vec8 gl = load_gain(gain_l, h, D, j);
             // local branch: dy = dO * wl; dx = r g dy - x r^3 mean(x g dy)
             float ss = 0.f, xgdy = 0.f;
@@ -223,6 +310,11 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
                     for (int i = 0; i < 8; ++i) accG[k][i] += g.v[i] * pt * xg.v[i] * r_g;
                 }
             }
+        }
+        if constexpr (UNIT) {
+            float lo, hi;
+            f2_unpack(dp2, lo, hi);
+            dp_acc = lo + hi;
         }
         // dp_t = z_t * sum_{h,d} dO (o~G - o~L); z_t is uniform over the block
         if (sel) {
@@ -277,13 +369,21 @@ int64_t wave_blocks(K kernel, int64_t ntok)
     return ntok < cap ? ntok : cap;
 }
 
+// Blocks of the gain-gradient backward (one partial row each): the larger of
+// its two variants, so the workspace fits whichever runs.
 int64_t gains_blocks(const logo_dims& d)
 {
     const int64_t ntok = static_cast<int64_t>(d.B) * d.T;
     switch (vec_per_thread(d)) {
-        case 1: return wave_blocks(combine_bwd_kernel<1, true>, ntok);
-        case 2: return wave_blocks(combine_bwd_kernel<2, true>, ntok);
-        default: return wave_blocks(combine_bwd_kernel<4, true>, ntok);
+        case 1:
+            return std::max(wave_blocks(combine_bwd_kernel<1, true, false>, ntok),
+                            wave_blocks(combine_bwd_kernel<1, true, true>, ntok));
+        case 2:
+            return std::max(wave_blocks(combine_bwd_kernel<2, true, false>, ntok),
+                            wave_blocks(combine_bwd_kernel<2, true, true>, ntok));
+        default:
+            return std::max(wave_blocks(combine_bwd_kernel<4, true, false>, ntok),
+                            wave_blocks(combine_bwd_kernel<4, true, true>, ntok));
     }
 }
 
@@ -317,14 +417,24 @@ extern "C" int logo_combine(const logo_bf16* o_l, const logo_bf16* o_c, const fl
         return LOGO_ERR_UNSUPPORTED;
     const int64_t ntok = static_cast<int64_t>(dims.B) * dims.T;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-#define LOGO_COMBINE_FWD(V)                                                                                       \
-    combine_fwd_kernel<V><<<static_cast<unsigned>(wave_blocks(combine_fwd_kernel<V>, ntok)), kThreads, 0, st>>>( \
-        o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, o, rstd_l, rstd_g, ntok, dims.Hq, dims.D)
-    switch (vec_per_thread(dims)) {
-        case 1: LOGO_COMBINE_FWD(1); break;
-        case 2: LOGO_COMBINE_FWD(2); break;
-        case 4: LOGO_COMBINE_FWD(4); break;
-        default: LOGO_COMBINE_FWD(8); break;
+#define LOGO_COMBINE_FWD(V, U)                                                                                 \
+    combine_fwd_kernel<V, U><<<static_cast<unsigned>(wave_blocks(combine_fwd_kernel<V, U>, ntok)), kThreads, 0, \
+                               st>>>(o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, o, rstd_l, rstd_g, ntok,    \
+                                     dims.Hq, dims.D)
+    if (!gain_l && !gain_g) {
+        switch (vec_per_thread(dims)) {
+            case 1: LOGO_COMBINE_FWD(1, true); break;
+            case 2: LOGO_COMBINE_FWD(2, true); break;
+            case 4: LOGO_COMBINE_FWD(4, true); break;
+            default: LOGO_COMBINE_FWD(8, true); break;
+        }
+    } else {
+        switch (vec_per_thread(dims)) {
+            case 1: LOGO_COMBINE_FWD(1, false); break;
+            case 2: LOGO_COMBINE_FWD(2, false); break;
+            case 4: LOGO_COMBINE_FWD(4, false); break;
+            default: LOGO_COMBINE_FWD(8, false); break;
+        }
     }
 #undef LOGO_COMBINE_FWD
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
@@ -354,22 +464,36 @@ int combine_bwd_common(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf1
     unsigned grid = 0;
     float* part = static_cast<float*>(workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-#define LOGO_COMBINE_BWD(V, G)                                                                                  \
-    grid = static_cast<unsigned>(wave_blocks(combine_bwd_kernel<V, G>, ntok));                                   \
-    combine_bwd_kernel<V, G><<<grid, kThreads, 0, st>>>(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, \
-                                                        dO_c, dgate_p, part, ntok, dims.Hq, dims.D)
-    if (gains) {
+#define LOGO_COMBINE_BWD(V, G, U)                                                                                 \
+    grid = static_cast<unsigned>(wave_blocks(combine_bwd_kernel<V, G, U>, ntok));                                  \
+    combine_bwd_kernel<V, G, U><<<grid, kThreads, 0, st>>>(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, \
+                                                           dO_c, dgate_p, part, ntok, dims.Hq, dims.D)
+    const bool unit = !gain_l && !gain_g;
+    if (gains && unit) {
         switch (vpt) {
-            case 1: LOGO_COMBINE_BWD(1, true); break;
-            case 2: LOGO_COMBINE_BWD(2, true); break;
-            default: LOGO_COMBINE_BWD(4, true); break;
+            case 1: LOGO_COMBINE_BWD(1, true, true); break;
+            case 2: LOGO_COMBINE_BWD(2, true, true); break;
+            default: LOGO_COMBINE_BWD(4, true, true); break;
+        }
+    } else if (gains) {
+        switch (vpt) {
+            case 1: LOGO_COMBINE_BWD(1, true, false); break;
+            case 2: LOGO_COMBINE_BWD(2, true, false); break;
+            default: LOGO_COMBINE_BWD(4, true, false); break;
+        }
+    } else if (unit) {
+        switch (vpt) {
+            case 1: LOGO_COMBINE_BWD(1, false, true); break;
+            case 2: LOGO_COMBINE_BWD(2, false, true); break;
+            case 4: LOGO_COMBINE_BWD(4, false, true); break;
+            default: LOGO_COMBINE_BWD(8, false, true); break;
         }
     } else {
         switch (vpt) {
-            case 1: LOGO_COMBINE_BWD(1, false); break;
-            case 2: LOGO_COMBINE_BWD(2, false); break;
-            case 4: LOGO_COMBINE_BWD(4, false); break;
-            default: LOGO_COMBINE_BWD(8, false); break;
+            case 1: LOGO_COMBINE_BWD(1, false, false); break;
+            case 2: LOGO_COMBINE_BWD(2, false, false); break;
+            case 4: LOGO_COMBINE_BWD(4, false, false); break;
+            default: LOGO_COMBINE_BWD(8, false, false); break;
         }
     }
 #undef LOGO_COMBINE_BWD
