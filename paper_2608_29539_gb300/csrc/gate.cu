@@ -17,6 +17,7 @@
 
 #include "colsum.cuh"
 #include "host_common.h"
+#include "sm100.cuh"
 
 namespace logo {
 namespace {
@@ -45,6 +46,9 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8])
     return raw;
 }
 
+// x_t . w for two tokens of a warp per pass (t and t + the warp count): one
+// load of w serves both, and two f32x2 chains per token keep the FMA
+// dependency chain a quarter as long as one scalar accumulator's.
 __global__ void __launch_bounds__(kFwdThreads) gate_fwd_kernel(const logo_bf16* __restrict__ x,
                                                                const float* __restrict__ w, int64_t ntok, int dm,
                                                                float* __restrict__ p)
@@ -53,27 +57,45 @@ __global__ void __launch_bounds__(kFwdThreads) gate_fwd_kernel(const logo_bf16* 
     const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kFwdThreads / 32);
     const int nv = dm / 8;
     for (int64_t t = static_cast<int64_t>(blockIdx.x) * (kFwdThreads / 32) + (threadIdx.x >> 5); t < ntok;
-         t += nwarps) {
+         t += 2 * nwarps) {
+        const int64_t t2 = t + nwarps;
+        const bool two = t2 < ntok;
         const uint4* xr = reinterpret_cast<const uint4*>(x + t * dm);
-        float a = 0.f;
+        const uint4* xr2 = reinterpret_cast<const uint4*>(x + (two ? t2 : t) * dm);
+        uint64_t a0 = 0ull, a1 = 0ull, b0 = 0ull, b1 = 0ull;
 #pragma unroll 4
         for (int v = lane; v < nv; v += 32) {
-            float xf[8];
-            unpack8(xr[v], xf);
             const float4* wv = reinterpret_cast<const float4*>(w + v * 8);
             const float4 w0 = __ldg(wv), w1 = __ldg(wv + 1);
-            a = fmaf(xf[0], w0.x, a);
-            a = fmaf(xf[1], w0.y, a);
-            a = fmaf(xf[2], w0.z, a);
-            a = fmaf(xf[3], w0.w, a);
-            a = fmaf(xf[4], w1.x, a);
-            a = fmaf(xf[5], w1.y, a);
-            a = fmaf(xf[6], w1.z, a);
-            a = fmaf(xf[7], w1.w, a);
+            const uint64_t wa = f2_pack(w0.x, w0.y), wb = f2_pack(w0.z, w0.w);
+            const uint64_t wc = f2_pack(w1.x, w1.y), wd = f2_pack(w1.z, w1.w);
+            float xf[8];
+            unpack8(xr[v], xf);
+            a0 = f2_fma(f2_pack(xf[0], xf[1]), wa, a0);
+            a1 = f2_fma(f2_pack(xf[2], xf[3]), wb, a1);
+            a0 = f2_fma(f2_pack(xf[4], xf[5]), wc, a0);
+            a1 = f2_fma(f2_pack(xf[6], xf[7]), wd, a1);
+            if (two) {
+                unpack8(xr2[v], xf);
+                b0 = f2_fma(f2_pack(xf[0], xf[1]), wa, b0);
+                b1 = f2_fma(f2_pack(xf[2], xf[3]), wb, b1);
+                b0 = f2_fma(f2_pack(xf[4], xf[5]), wc, b0);
+                b1 = f2_fma(f2_pack(xf[6], xf[7]), wd, b1);
+            }
         }
+        float u0, u1, u2, u3;
+        f2_unpack(f2_add(a0, a1), u0, u1);
+        f2_unpack(f2_add(b0, b1), u2, u3);
+        float a = u0 + u1, b = u2 + u3;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-        if (lane == 0) p[t] = 1.0f / (1.0f + expf(-a));
+        for (int o = 16; o > 0; o >>= 1) {
+            a += __shfl_xor_sync(0xffffffffu, a, o);
+            b += __shfl_xor_sync(0xffffffffu, b, o);
+        }
+        if (lane == 0) {
+            p[t] = 1.0f / (1.0f + expf(-a));
+            if (two) p[t2] = 1.0f / (1.0f + expf(-b));
+        }
     }
 }
 
