@@ -91,6 +91,18 @@ LOGO_API int logo_get_device_status(int* status);
  * current context); informational. */
 LOGO_API int logo_num_sms(void);
 
+/* Self-test of the bounded device waits (no counterpart in the paper).  Every
+ * pipelined kernel waits on shared-memory mbarriers with a wall-clock budget
+ * (2 s); when a budget runs out the kernel records LOGO_ERR_TIMEOUT, stops its
+ * roles and returns, so a lost arrival becomes a status instead of a hang.
+ * This call launches one warp that waits, through that same wait, on an
+ * mbarrier nothing will ever arrive at, with a budget of budget_ns
+ * nanoseconds (1 .. 2e9).  After it completes, logo_get_device_status()
+ * reports LOGO_ERR_TIMEOUT, and the context remains usable.  No device fault
+ * or trap is involved.  Returns LOGO_ERR_INVALID_ARG for a budget out of
+ * range, LOGO_ERR_CUDA if the launch fails. */
+LOGO_API int logo_selftest_wait_expiry(uint64_t budget_ns, void* stream);
+
 /* ------------------------------------------------------------------------
  * logo_select -- routing decision and packing of the selected set.
  *   Eq. 7 (Sec. 3.2): z_t = 1[p_t > b_th], the gate p_t = sigmoid(x_t . w_g)

@@ -208,6 +208,8 @@ int check_gate(const logo_dims& d, int dm)
 }
 
 }  // namespace
+int gate_tu_status(int clear) { return read_tu_status(clear); }
+
 }  // namespace logo
 
 using namespace logo;

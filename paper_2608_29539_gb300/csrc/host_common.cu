@@ -72,8 +72,9 @@ extern "C" int logo_get_device_status(int* status)
 {
     if (!status) return LOGO_ERR_INVALID_ARG;
     int first = LOGO_OK;
-    int (*readers[])(int) = {logo::select_tu_status, logo::combine_tu_status, logo::attn_fwd_tu_status,
-                             logo::attn_bwd_tu_status, logo::decode_tu_status};
+    int (*readers[])(int) = {logo::select_tu_status,    logo::combine_tu_status,   logo::attn_fwd_tu_status,
+                             logo::attn_bwd_tu_status,  logo::decode_tu_status,    logo::transform_tu_status,
+                             logo::gate_tu_status,      logo::selftest_tu_status};
     for (auto rd : readers) {
         int v = rd(1);
         if (v == LOGO_ERR_CUDA) return LOGO_ERR_CUDA;

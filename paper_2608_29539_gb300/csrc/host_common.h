@@ -40,5 +40,8 @@ int combine_tu_status(int clear);
 int attn_fwd_tu_status(int clear);
 int attn_bwd_tu_status(int clear);
 int decode_tu_status(int clear);
+int transform_tu_status(int clear);
+int gate_tu_status(int clear);
+int selftest_tu_status(int clear);
 
 }  // namespace logo

@@ -89,7 +89,8 @@ constexpr uint64_t kWaitBudgetNs = 2000000000ull;
 // Wait for the phase with the given parity to complete.  Returns false (after
 // recording a timeout) if the budget runs out or another role of the CTA has
 // already aborted; the caller then stops issuing work.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag)
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          uint64_t budget_ns = kWaitBudgetNs)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
@@ -97,7 +98,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63u) == 0) {
             if (*abort_flag) return false;
-            if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+            if (globaltimer_ns() - t0 > budget_ns) {
                 *abort_flag = 1;
                 record_status(LOGO_ERR_TIMEOUT);
                 return false;

@@ -786,6 +786,8 @@ int launch_lp_bwd(const logo_bf16* u_l, const logo_bf16* a, const logo_bf16* du_
 }
 
 }  // namespace
+int transform_tu_status(int clear) { return read_tu_status(clear); }
+
 }  // namespace logo
 
 using namespace logo;

@@ -55,6 +55,7 @@ _lib = None
 _SIGS = {
     "logo_get_device_status": (_c_int, [ctypes.POINTER(_c_int)]),
     "logo_num_sms": (_c_int, []),
+    "logo_selftest_wait_expiry": (_c_int, [ctypes.c_uint64, _vp]),
     "logo_select_workspace_size": (_c_size, [Dims]),
     "logo_select": (_c_int, [_vp, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp, _c_size, _vp]),
     "logo_gate_select": (_c_int, [_vp, _vp, _c_int, Dims, _c_int, _c_float, _c_float, _vp, _vp, _vp, _vp, _vp, _vp,
@@ -167,6 +168,12 @@ def logo_get_device_status() -> int:
 
 def logo_num_sms() -> int:
     return int(lib().logo_num_sms())
+
+
+def logo_selftest_wait_expiry(budget_ns: int) -> None:
+    """Launch one warp whose bounded mbarrier wait can never complete; after
+    budget_ns it records LOGO_ERR_TIMEOUT (read it with logo_get_device_status)."""
+    _call("logo_selftest_wait_expiry", int(budget_ns), _stream())
 
 
 def logo_select(gate_p, mode: int, b_th: float = 0.5, ratio: float = 0.0, z=None, pos=None, cu_q=None,

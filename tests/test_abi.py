@@ -216,3 +216,12 @@ def test_workspace_sizes_grow_with_shape(lib):
         if fn != "logo_select_workspace_size":
             assert a < b, fn
     assert L.logo_global_attn_fwd_workspace_size(logo.Dims(1, 128, 2, 2, 96)) == 0
+
+
+def test_wait_expiry_selftest_host_checks(lib):
+    from paper_2608_29539_gb300 import logo
+    L = lib
+    L.logo_selftest_wait_expiry.restype = ctypes.c_int
+    L.logo_selftest_wait_expiry.argtypes = [ctypes.c_uint64, ctypes.c_void_p]
+    assert L.logo_selftest_wait_expiry(0, None) == logo.LOGO_ERR_INVALID_ARG
+    assert L.logo_selftest_wait_expiry(2_000_000_001, None) == logo.LOGO_ERR_INVALID_ARG
