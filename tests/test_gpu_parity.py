@@ -225,7 +225,12 @@ COMBINE_CASES = [
     (1, 513, 3, 64, 0.5, False),
     (2, 100, 2, 128, 0.0, True),
     (1, 64, 2, 64, 1.0, True),
+    (1, 200, 32, 128, 0.125, False),  # unit gains, two vectors per thread (the 16K workload's width)
+    (1, 100, 64, 128, 0.25, False),   # unit gains, four vectors per thread
 ]
+# the widest rows the combine accepts (Hq*D = 16384, eight vectors per thread);
+# beyond the gain-gradient variant's limit, so forward and backward only
+WIDE_CASES = [(1, 50, 128, 128, 0.5, False), (1, 40, 128, 128, 0.5, True)]
 
 
 def _combine_setup(B, T, H, D, ratio, gains, seed):
@@ -240,7 +245,7 @@ def _combine_setup(B, T, H, D, ratio, gains, seed):
     return p, (z, row_of), nn, o_l, o_c, gl, gg
 
 
-@pytest.mark.parametrize("B,T,H,D,ratio,gains", COMBINE_CASES)
+@pytest.mark.parametrize("B,T,H,D,ratio,gains", COMBINE_CASES + WIDE_CASES)
 def test_combine_fwd(B, T, H, D, ratio, gains):
     p, (z, row_of), n, o_l, o_c, gl, gg = _combine_setup(B, T, H, D, ratio, gains, seed=T)
     cu = lambda t: None if t is None else t.cuda()  # noqa: E731
@@ -255,7 +260,7 @@ def test_combine_fwd(B, T, H, D, ratio, gains):
         check_close(np32(rg)[:n], rrg, "rstd_g", 1e-5, 1e-5)
 
 
-@pytest.mark.parametrize("B,T,H,D,ratio,gains", COMBINE_CASES)
+@pytest.mark.parametrize("B,T,H,D,ratio,gains", COMBINE_CASES + WIDE_CASES)
 def test_combine_bwd(B, T, H, D, ratio, gains):
     p, (z, row_of), n, o_l, o_c, gl, gg = _combine_setup(B, T, H, D, ratio, gains, seed=2 * T)
     dO = seeded((B, T, H, D), 5 * T, torch.bfloat16)
