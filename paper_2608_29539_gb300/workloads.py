@@ -62,10 +62,12 @@ def sweep(ratio: float) -> Workload:
                     ratio=ratio, seed=4)
 
 
-def clustered_logits(T: int, gen: torch.Generator, mean_run: float = 16.0, frac: float = 0.125):
-    """Gate logits with clustered high values: a two-state Markov chain whose
-    'on' runs have mean length ``mean_run`` and stationary share ``frac``; the
-    logit is N(0,1) + 4 * state."""
+def clustered_states(T: int, gen: torch.Generator, mean_run: float = 16.0, frac: float = 0.125) -> torch.Tensor:
+    """The on/off states behind clustered gates: a two-state Markov chain whose
+    'on' runs have mean length ``mean_run`` (leave with probability 1/mean_run)
+    and whose stationary 'on' share is ``frac`` (enter with probability
+    (1/mean_run) * frac / (1 - frac)); the first state is drawn from the
+    stationary distribution.  Returns float32 0/1 of length T."""
     p_off = 1.0 / mean_run
     p_on = p_off * frac / (1.0 - frac)
     u = torch.rand(T, generator=gen, dtype=torch.float64)
@@ -79,7 +81,13 @@ def clustered_logits(T: int, gen: torch.Generator, mean_run: float = 16.0, frac:
             elif s == 0 and ul[t] < p_on:
                 s = 1
         st[t] = float(s)
-    state = torch.tensor(st, dtype=torch.float32)
+    return torch.tensor(st, dtype=torch.float32)
+
+
+def clustered_logits(T: int, gen: torch.Generator, mean_run: float = 16.0, frac: float = 0.125):
+    """Gate logits with clustered high values: N(0,1) + 4 * state, the state
+    from ``clustered_states`` (drawn first, then the noise)."""
+    state = clustered_states(T, gen, mean_run, frac)
     noise = torch.randn(T, generator=gen, dtype=torch.float32)
     return noise + 4.0 * state
 
