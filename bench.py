@@ -593,10 +593,11 @@ def native_arm(a, rank, world, local_rank, dist_on):
     kernel_src = os.path.join(ROOT, "paper_2608_29539_gb300", "csrc",
                               "attn_bwd.cu" if dom.endswith("bwd") else "attn_fwd.cu")
     tr = TRAFFIC.get((dom, src_hash(kernel_src)))
-    roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-            "frac": achieved / pk["bf16_sus"], "traffic": tr,
-            "peak_note": f"{pk['src']} sustained bf16 (kernel timed inside a multi-ms step); "
-                         f"frac of burst peak {achieved / pk['bf16']:.3f}",
+    roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+            "frac": achieved / pk["bf16"], "traffic": tr,
+            "peak_note": f"{pk['src']} burst bf16 (the call runs for about a millisecond at the maximum SM "
+                         f"clock); frac of the sustained peak {achieved / pk['bf16_sus']:.3f}",
+            "frac_of_sustained": achieved / pk["bf16_sus"],
             "timing": "CUDA events around the call on its launching stream, mean over K eager steps"}
     l_ms = per_call["local_fwd"] + per_call["local_bwd"]
     breakdown = {c: {"ms": per_call[c]} for c in CALLS}
@@ -605,9 +606,11 @@ def native_arm(a, rank, world, local_rank, dist_on):
     line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": a.steps,
             "warmup": a.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded; no dataset)", "config": config_of(w),
-            "frac_of_peak": value / pk["bf16_sus"],
+            "frac_of_peak": value / pk["bf16"], "frac_of_sustained_peak": value / pk["bf16_sus"],
             "global_fwd_bwd": {"tflops": fl_global / (g_ms / 1e3) / 1e12,
-                               "frac_of_peak": fl_global / (g_ms / 1e3) / 1e12 / pk["bf16_sus"], "ms": g_ms},
+                               "frac_of_peak": fl_global / (g_ms / 1e3) / 1e12 / pk["bf16"],
+                               "frac_of_sustained_peak": fl_global / (g_ms / 1e3) / 1e12 / pk["bf16_sus"],
+                               "ms": g_ms},
             "local_fwd_bwd": {"tflops": fl_local / (l_ms / 1e3) / 1e12, "ms": l_ms},
             "useful_flops_per_step": fl_step, "pairs_per_head": {"local": lp, "global": gp},
             "selected": n, "per_call": breakdown, "roofline": roof,

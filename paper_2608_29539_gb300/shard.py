@@ -72,7 +72,12 @@ def all_reduce_gate_grad(dgate: torch.Tensor, process_group=None) -> torch.Tenso
     """Sum the per-rank partial dp over the head shards, in place."""
     import torch.distributed as dist
     if dist.is_available() and dist.is_initialized() and dist.get_world_size(process_group) > 1:
-        dist.all_reduce(dgate, op=dist.ReduceOp.SUM, group=process_group)
+        if dgate.is_cuda and dist.get_backend(process_group) == "gloo":
+            host = dgate.cpu()  # gloo reduces host memory; the vector is B*T floats
+            dist.all_reduce(host, op=dist.ReduceOp.SUM, group=process_group)
+            dgate.copy_(host)
+        else:
+            dist.all_reduce(dgate, op=dist.ReduceOp.SUM, group=process_group)
     return dgate
 
 
