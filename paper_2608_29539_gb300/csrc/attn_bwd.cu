@@ -7,23 +7,39 @@
 // gradient and Dsum = rowsum(dO * O):
 //   dV = P^T dO,  dP = dO V^T,  dS = P * (dP - Dsum),
 //   dQ = scale * dS K,  dK = scale * dS^T Q.
-// One persistent kernel template serves both branches.  Work items are KV
-// blocks (128 keys of one KV head of one sequence); an item walks every
-// (query head of the KV head's group) x (query tile that can see the block).
-// For the global branch the query tiles are 128-row slices of the packed
-// selected rows, and a binary search over the packed positions finds the
-// first row that can see the block (the precomputed search of App. B): no
-// earlier tile is visited.  Per (query tile, KV block):
-//   MMA warp      S^T = K Q^T and dP^T = V dO^T into TMEM; after the softmax
-//                 warps have written P^T and dS^T (bf16) to shared memory:
-//                 dV += P^T dO, dK += dS^T Q (TMEM accumulators for the whole
-//                 item) and dQ = dS K into the S^T columns.
-//   4 warps       thread = key row: P^T and dS^T from S^T, dP^T and the
-//                 per-query lse / Dsum; then thread = query row: dQ out of
-//                 TMEM, added into an fp32 accumulator with vector atomics.
-//   TMA warp      K/V once per item, Q/dO per tile.
-// Five MMAs per tile pair (the minimum); dK/dV need no atomics because one
-// CTA owns a KV block for all query heads of its group.
+// Both kernels are persistent and KV-block-major: a work item is one block of
+// 128 keys of one KV head of one sequence, and it walks every (query head of
+// the KV head's group) x (query tile that can see the block).  dK and dV stay
+// in TMEM for the whole item (one CTA owns the block for every query head of
+// its group, so they need no atomics); dQ is reduced across items in fp32.
+// Five MMAs per (query tile, KV block), the minimum: the paper's separate dQ
+// and dK/dV kernels recompute S and dP and take seven.
+//
+// d = 128, attn_bwd2_kernel (16 warps, query tiles of 64 rows):
+//   warp 0       TMA: K/V once per item, Q/dO tiles through a 4-deep ring
+//   warp 1       MMA issuer A: S^T = K Q^T, dP^T = V dO^T (M = 128 keys,
+//                N = 64 queries) into one TMEM buffer that the softmax warps
+//                release as soon as they have loaded it
+//   warps 2..9   two warpgroups, one per 32-query half of the tile; thread =
+//                key row: P^T (back to TMEM as bf16 pairs, two buffers) and
+//                dS^T (bf16, to shared memory, two buffers)
+//   warp 15      MMA issuer B: dV += P^T dO (P^T as the TMEM operand),
+//                dK += dS^T Q, dQ^T = K^T dS^T into a TMEM buffer of its own
+//   warps 10..13 dQ^T out of TMEM (thread = head-dim row), coalesced fp32
+//                reductions into the dQ accumulator (one 128-byte row segment
+//                per warp instruction), converted to bf16 by a pass after the
+//                kernel; dK/dV epilogue at the end of each item
+//   warp 14      global branch: zero rows of the dense dQ for unselected tokens
+// Global query tiles are 64-row slices of the packed selected rows, starting
+// at the first packed row whose position reaches the block, read from a table
+// the pre-pass builds once per call (App. B's precomputed search); the same
+// pre-pass gathers the selected Q rows and computes Dsum.
+//
+// d = 64, attn_bwd_kernel (6 warps, query tiles of 128 rows): one MMA warp
+// issues S^T, dP^T, then dV, dK and dQ into the S^T columns once the softmax
+// warps have written P^T and dS^T to shared memory; the first visible query
+// tile of a global item comes from a binary search over the packed positions;
+// dQ goes through fp32 atomics and a conversion pass.
 #include <cuda_bf16.h>
 
 #include <cstdint>
