@@ -210,9 +210,11 @@ LOGO_API int logo_decode_global_sparse_attn(const logo_bf16* q, const logo_bf16*
  *   Limits: B <= LOGO_SELECT_NOALLOC_MAX_SEQS and B * ceil(T / 1024) <=
  *   LOGO_SELECT_NOALLOC_MAX_CHUNKS (at most 16,777,216 tokens per call);
  *   larger shapes return LOGO_ERR_SCRATCH_LIMIT before anything is launched.
- *   The first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress, with that device current): make that first call
- *   before any stream capture.  All calls share the one array, which keeps
+ *   The first call in each CUDA context looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current) and caches it under the
+ *   context's id: make that first call before any stream capture, and again
+ *   after anything that recreates the context (cudaDeviceReset), which the
+ *   next call notices and repeats the lookup for.  All calls share the one array, which keeps
  *   the previous call's contents; every kernel writes the scratch it reads
  *   before reading it, so no clearing is needed, but calls that overlap on
  *   the GPU (different streams, or concurrent host threads) race on it and

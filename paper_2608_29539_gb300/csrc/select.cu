@@ -584,21 +584,58 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_select_noalloc_scratch[LOGO_SELECT_NOALLOC_SCRATCH_BYTES];
 
-// Device address of the array, looked up once per device (the name is only a
-// host-side stand-in and must never be passed to a kernel).
+// Id of the calling thread's current CUDA context (0 when there is none yet
+// or the driver cannot tell), through the driver entry points, so the
+// library keeps no link-time dependency on libcuda.
+unsigned long long current_context_id()
+{
+    typedef CUresult (*GetCurrentFn)(CUcontext*);
+    typedef CUresult (*GetIdFn)(CUcontext, unsigned long long*);
+    static GetCurrentFn get_current = nullptr;
+    static GetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<GetCurrentFn>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<GetIdFn>(p);
+    });
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+        return 0;
+    return id;
+}
+
+// Device address of the array in the current context (the name is only a
+// host-side stand-in and must never be passed to a kernel).  Looked up on the
+// first call in each context and cached under the context's id, so a context
+// that was destroyed and created again (cudaDeviceReset) gets a fresh lookup
+// instead of a stale address.  Without a context id the lookup is repeated on
+// every call.
 int noalloc_scratch_ptr(char** out)
 {
     static std::mutex mu;
-    static void* cached[64] = {nullptr};
+    static unsigned long long cached_ctx[64] = {0};
+    static void* cached_ptr[64] = {nullptr};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return LOGO_ERR_CUDA;
     std::lock_guard<std::mutex> lock(mu);
-    if (!cached[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_select_noalloc_scratch) != cudaSuccess || !p) return LOGO_ERR_CUDA;
-        cached[dev] = p;
+    const unsigned long long ctx = current_context_id();
+    if (ctx != 0 && ctx == cached_ctx[dev] && cached_ptr[dev]) {
+        *out = static_cast<char*>(cached_ptr[dev]);
+        return LOGO_OK;
     }
-    *out = static_cast<char*>(cached[dev]);
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_select_noalloc_scratch) != cudaSuccess || !p) return LOGO_ERR_CUDA;
+    cached_ctx[dev] = current_context_id();  // the lookup creates the context if there was none
+    cached_ptr[dev] = p;
+    *out = static_cast<char*>(p);
     return LOGO_OK;
 }
 
