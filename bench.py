@@ -173,40 +173,69 @@ def launches_per_step(w):
     return n
 
 
-def run_step(layer, g, ev=None):
-    """One full step; if ev is given, record an event after each call."""
+def step_calls(layer, g):
+    """The seven calls of one step, in order, as (name, thunk) pairs."""
     from paper_2608_29539_gb300 import logo as L
     c = layer.cfg
+    return [
+        ("select", lambda: L.logo_select(g["p"], c.mode, c.b_th, c.ratio, layer.z, layer.pos, layer.cu_q,
+                                         layer.row_of, layer.n_sel, workspace=layer.ws)),
+        ("local_fwd", lambda: L.logo_local_attn_fwd(g["qL"], g["kL"], g["vL"], c.window, c.scale, layer.o_l,
+                                                    layer.lse_l)),
+        ("global_fwd", lambda: L.logo_global_sparse_attn_fwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q,
+                                                             layer.n_sel, c.scale, layer.o_c, layer.lse_c,
+                                                             workspace=layer.ws)),
+        ("combine", lambda: L.logo_combine(layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of, None, None, c.eps,
+                                           layer.o, layer.rstd_l, layer.rstd_g)),
+        ("combine_bwd", lambda: L.logo_combine_bwd(g["dO"], layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of,
+                                                   None, None, c.eps, layer.dO_l, layer.dO_c, layer.dgate)),
+        ("global_bwd", lambda: L.logo_global_sparse_attn_bwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q,
+                                                             layer.n_sel, layer.o_c, layer.lse_c, layer.dO_c,
+                                                             c.scale, layer.dqG, layer.dkG, layer.dvG,
+                                                             workspace=layer.ws)),
+        ("local_bwd", lambda: L.logo_local_attn_bwd(g["qL"], g["kL"], g["vL"], layer.o_l, layer.lse_l, layer.dO_l,
+                                                    c.window, c.scale, layer.dqL, layer.dkL, layer.dvL,
+                                                    workspace=layer.ws)),
+    ]
+
+
+def run_step(layer, g, ev=None):
+    """One full step; if ev is given, record an event after each call."""
     if ev is not None:
         ev[0].record()
-    L.logo_select(g["p"], c.mode, c.b_th, c.ratio, layer.z, layer.pos, layer.cu_q, layer.row_of, layer.n_sel,
-                  workspace=layer.ws)
-    if ev is not None:
-        ev[1].record()
-    L.logo_local_attn_fwd(g["qL"], g["kL"], g["vL"], c.window, c.scale, layer.o_l, layer.lse_l)
-    if ev is not None:
-        ev[2].record()
-    L.logo_global_sparse_attn_fwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q, layer.n_sel, c.scale,
-                                  layer.o_c, layer.lse_c, workspace=layer.ws)
-    if ev is not None:
-        ev[3].record()
-    L.logo_combine(layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of, None, None, c.eps, layer.o, layer.rstd_l,
-                   layer.rstd_g)
-    if ev is not None:
-        ev[4].record()
-    L.logo_combine_bwd(g["dO"], layer.o_l, layer.o_c, g["p"], layer.z, layer.row_of, None, None, c.eps,
-                       layer.dO_l, layer.dO_c, layer.dgate)
-    if ev is not None:
-        ev[5].record()
-    L.logo_global_sparse_attn_bwd(g["qG"], g["kG"], g["vG"], layer.pos, layer.cu_q, layer.n_sel, layer.o_c,
-                                  layer.lse_c, layer.dO_c, c.scale, layer.dqG, layer.dkG, layer.dvG,
-                                  workspace=layer.ws)
-    if ev is not None:
-        ev[6].record()
-    L.logo_local_attn_bwd(g["qL"], g["kL"], g["vL"], layer.o_l, layer.lse_l, layer.dO_l, c.window, c.scale,
-                          layer.dqL, layer.dkL, layer.dvL, workspace=layer.ws)
-    if ev is not None:
-        ev[7].record()
+    for i, (_, call) in enumerate(step_calls(layer, g)):
+        call()
+        if ev is not None:
+            ev[i + 1].record()
+
+
+def per_call_device_ms(layer, g, reps):
+    """Device time of each call: the call captured `reps` times back to back as
+    one CUDA graph, one replay timed with CUDA events on the launching stream,
+    divided by `reps`.  (Timing single eager calls would add the host's launch
+    time of a small call to its duration.)  Every call is idempotent on the
+    step's buffers, so repeating it leaves the state of the step unchanged."""
+    out = {}
+    for name, call in step_calls(layer, g):
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            call()
+        torch.cuda.current_stream().wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for _ in range(reps):
+                call()
+        graph.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        out[name] = e0.elapsed_time(e1) / reps
+        del graph
+    return out
 
 
 def layer_for(w, device):
@@ -578,9 +607,10 @@ def native_arm(a, rank, world, local_rank, dist_on):
     total_ms = t_start.elapsed_time(t_end)
     total_ms = max_over_ranks(total_ms, dist_on)
     ms_step = total_ms / a.steps
-    per_call = {c: float(np.mean([evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(a.steps)]))
-                for i, c in enumerate(CALLS)}
+    per_call_eager = {c: float(np.mean([evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(a.steps)]))
+                      for i, c in enumerate(CALLS)}
     eager_ms = float(np.mean([evs[s][0].elapsed_time(evs[s][7]) for s in range(a.steps)]))
+    per_call = per_call_device_ms(layer, x, reps=max(3, a.steps))
     flops_all = sum_over_ranks(fl_step * a.steps, dist_on)
     value = flops_all / (total_ms / 1e3) / 1e12
 
@@ -598,9 +628,10 @@ def native_arm(a, rank, world, local_rank, dist_on):
             "peak_note": f"{pk['src']} burst bf16 (the call runs for about a millisecond at the maximum SM "
                          f"clock); frac of the sustained peak {achieved / pk['bf16_sus']:.3f}",
             "frac_of_sustained": achieved / pk["bf16_sus"],
-            "timing": "CUDA events around the call on its launching stream, mean over K eager steps"}
+            "timing": "CUDA events on the launching stream around one replay of a CUDA graph holding the "
+                      "call K times back to back, divided by K"}
     l_ms = per_call["local_fwd"] + per_call["local_bwd"]
-    breakdown = {c: {"ms": per_call[c]} for c in CALLS}
+    breakdown = {c: {"ms": per_call[c], "ms_eager_call": per_call_eager[c]} for c in CALLS}
     for c, fl in flops_call.items():
         breakdown[c]["tflops"] = fl / (per_call[c] / 1e3) / 1e12
     line = {"metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": a.steps,

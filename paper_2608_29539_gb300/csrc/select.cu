@@ -12,6 +12,13 @@
 //                        cu_q[] and the total N.
 //   write_kernel         per chunk: block-wide prefix sums (warp ballots) turn
 //                        the decisions into z, pos and row_of, in ascending t.
+// Ratio mode with 4K < T <= 128K takes one launch instead:
+//   select_ratio_cluster_kernel  one 8-CTA cluster per sequence; the CTAs share
+//                        their radix histograms and counts through distributed
+//                        shared memory.  Up to 4K, select_ratio_small_kernel
+//                        (one block per sequence) does the same in one CTA.
+#include <cooperative_groups.h>
+
 #include <cstdint>
 #include <mutex>
 
@@ -339,6 +346,175 @@ __global__ void __launch_bounds__(1024) select_ratio_small_kernel(const float* _
     }
 }
 
+// Ratio mode, 4K < T <= kClusterCTAs * 1024 * KPT: one cluster of kClusterCTAs
+// CTAs per sequence (a thread-block cluster; grid = B clusters).  CTA r of the
+// cluster owns tokens [r C, r C + C), C = ceil(T / kClusterCTAs), thread i of it
+// the KPT consecutive tokens starting at r C + KPT i, kept in registers.  Each
+// radix pass counts the CTA's own keys into its 256-bin histogram (lanes with
+// the same bin grouped, one shared atomic per group), then every CTA sums all
+// kClusterCTAs histograms out of distributed shared memory, in rank order, and
+// picks the same bin.  Histograms alternate between two buffers, so one
+// cluster barrier per pass suffices: a buffer is cleared right after the
+// barrier that follows its last remote read.  Finally the CTAs exchange their
+// counts of keys above and equal to the threshold: tied keys are taken in
+// position order, so a CTA's first tied rank and its first packed row follow
+// from the counts of the CTAs before it.  Same decisions as the one-block
+// kernel, bit for bit.
+constexpr int kClusterCTAs = 8;
+
+template <int KPT>
+__global__ void __cluster_dims__(kClusterCTAs, 1, 1) __launch_bounds__(1024)
+    select_ratio_cluster_kernel(const float* __restrict__ p, int B, int T, int k, uint8_t* __restrict__ z,
+                                int32_t* __restrict__ pos, int32_t* __restrict__ cu_q,
+                                int32_t* __restrict__ row_of, int32_t* __restrict__ n_total)
+{
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    __shared__ int hist[2][256];        // this CTA's histogram of the pass (two buffers, read by the cluster)
+    __shared__ int ghist[256];          // the cluster's histogram of the pass
+    __shared__ int counts[2];           // keys above / equal to the threshold in this CTA (read by the cluster)
+    __shared__ uint32_t sh_prefix;
+    __shared__ int sh_remaining;
+    __shared__ int sh_warp[32];
+    __shared__ int sh_total;
+    const int rank = static_cast<int>(cluster.block_rank());
+    const int b = blockIdx.x / kClusterCTAs, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t off = static_cast<int64_t>(b) * T;
+    const int C = (T + kClusterCTAs - 1) / kClusterCTAs;
+    const int c0 = rank * C, c1 = min(T, c0 + C);
+    const int t0 = c0 + threadIdx.x * KPT;
+    uint32_t key[KPT];
+    bool valid[KPT];
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        valid[u] = t0 + u < c1;
+        key[u] = valid[u] ? gate_key(p[off + t0 + u]) : 0u;
+    }
+    if (threadIdx.x < 256) {
+        hist[0][threadIdx.x] = 0;
+        hist[1][threadIdx.x] = 0;
+    }
+    __syncthreads();
+    const int k_eff = k <= 0 ? 0 : (k >= T ? T : k);
+    uint32_t prefix = 0;
+    int remaining = k;
+    if (k <= 0) {
+        prefix = 0xFFFFFFFFu;
+        remaining = 0;
+    } else if (k >= T) {
+        prefix = 0u;
+        remaining = T;
+    } else {
+        uint32_t mask = 0;
+        int buf = 0;
+        for (int shift = 24; shift >= 0; shift -= 8, buf ^= 1) {
+#pragma unroll
+            for (int u = 0; u < KPT; ++u) {
+                const bool in = valid[u] && (key[u] & mask) == prefix;
+                const uint32_t bin = (key[u] >> shift) & 0xFFu;
+                const unsigned same = __match_any_sync(0xffffffffu, in ? bin : 0x100u);
+                if (in && lane == __ffs(same) - 1) atomicAdd(&hist[buf][bin], __popc(same));
+            }
+            cluster.sync();  // every CTA's histogram of this pass is complete
+            if (threadIdx.x < 256) {
+                int sum = 0;
+                for (int r = 0; r < kClusterCTAs; ++r) sum += cluster.map_shared_rank(&hist[buf][0], r)[threadIdx.x];
+                ghist[threadIdx.x] = sum;
+                // the other buffer was last read remotely before the barrier above
+                hist[buf ^ 1][threadIdx.x] = 0;
+            }
+            __syncthreads();
+            if (warp == 0) hist_pick(ghist, remaining, prefix, shift, &sh_prefix, &sh_remaining);
+            __syncthreads();
+            prefix = sh_prefix;
+            remaining = sh_remaining;
+            mask |= 0xFFu << shift;
+        }
+    }
+    // exclusive scan over the CTA's 1024 threads in order; the total to every thread
+    auto block_scan = [&](int v, int* total) {
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) sh_warp[warp] = x;
+        __syncthreads();
+        if (warp == 0) {
+            const int w0 = sh_warp[lane];
+            int w = w0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w += y;
+            }
+            sh_warp[lane] = w - w0;  // exclusive over warps
+            if (lane == 31) sh_total = w;
+        }
+        __syncthreads();
+        const int r = sh_warp[warp] + x - v;
+        *total = sh_total;
+        __syncthreads();
+        return r;
+    };
+    // this CTA's keys above the threshold (low 16 bits) and tied with it (high
+    // 16 bits; at most 16K per CTA), scanned together
+    int ngt = 0, neq = 0;
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        ngt += (valid[u] && key[u] > prefix) ? 1 : 0;
+        neq += (valid[u] && key[u] == prefix) ? 1 : 0;
+    }
+    int tot;
+    const int ex = block_scan(ngt | (neq << 16), &tot);
+    int eq_rank = ex >> 16;
+    if (threadIdx.x == 0) {
+        counts[0] = tot & 0xFFFF;
+        counts[1] = tot >> 16;
+    }
+    cluster.sync();  // every CTA's counts are published
+    // tied keys in earlier CTAs, and the packed rows the earlier CTAs fill
+    int eq_before = 0, rows_before = 0;
+    for (int r = 0; r < rank; ++r) {
+        const int* rc = cluster.map_shared_rank(&counts[0], r);
+        const int gt_r = rc[0], eq_r = rc[1];
+        rows_before += gt_r + max(0, min(eq_r, remaining - eq_before));
+        eq_before += eq_r;
+    }
+    eq_rank += eq_before;
+    bool sel[KPT];
+    int nsel = 0;
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        bool take = false;
+        if (valid[u] && key[u] == prefix) {
+            take = eq_rank < remaining;
+            ++eq_rank;
+        }
+        sel[u] = valid[u] && (key[u] > prefix || take);
+        nsel += sel[u];
+    }
+    int tot_sel;
+    int row = b * k_eff + rows_before + block_scan(nsel, &tot_sel);
+#pragma unroll
+    for (int u = 0; u < KPT; ++u) {
+        if (valid[u]) {
+            z[off + t0 + u] = sel[u] ? 1 : 0;
+            row_of[off + t0 + u] = sel[u] ? row : -1;
+            if (sel[u]) pos[row++] = t0 + u;
+        }
+    }
+    if (rank == 0 && threadIdx.x == 0) {
+        cu_q[b] = b * k_eff;
+        if (b == B - 1) {
+            cu_q[B] = B * k_eff;
+            *n_total = B * k_eff;
+        }
+    }
+    cluster.sync();  // no CTA leaves while another may still read its counts
+}
+
 struct ChunkCounts {
     int gt;   // tokens selected outright in the chunk
     int eq;   // tokens tied with the threshold key (ratio mode)
@@ -530,18 +706,29 @@ extern "C" int logo_select(const float* gate_p, logo_dims dims, int mode, float 
     const int nchunk = (dims.T + kChunk - 1) / kChunk;
     // k = floor(rho * T), with rho read as float32 and the product in double
     const int k = ratio_mode ? static_cast<int>(static_cast<double>(ratio) * dims.T) : 0;
-    if (ratio_mode && dims.T <= 16 * 1024) {  // one launch: one block per sequence
+    if (ratio_mode && dims.T <= 4 * 1024) {  // one launch: one block per sequence
         const int smem =
             static_cast<int>(round_up((static_cast<size_t>(dims.T) + dims.T / 16 + 1 + dims.T) * 4 + dims.T, 16));
-        if (dims.T <= 4 * 1024) {
-            if (set_smem_limit(select_ratio_small_kernel<4>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
-            select_ratio_small_kernel<4><<<dims.B, 1024, smem, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
-                                                                     n_sel_total);
-        } else {
-            if (set_smem_limit(select_ratio_small_kernel<16>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
-            select_ratio_small_kernel<16><<<dims.B, 1024, smem, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q,
-                                                                      row_of, n_sel_total);
-        }
+        if (set_smem_limit(select_ratio_small_kernel<4>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
+        select_ratio_small_kernel<4><<<dims.B, 1024, smem, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                 n_sel_total);
+        return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
+    }
+    if (ratio_mode && dims.T <= kClusterCTAs * 1024 * 16) {  // one launch: one 8-CTA cluster per sequence
+        const dim3 grid(dims.B * kClusterCTAs);
+        const int per_cta = (dims.T + kClusterCTAs - 1) / kClusterCTAs;
+        if (per_cta <= 2 * 1024)
+            select_ratio_cluster_kernel<2><<<grid, 1024, 0, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                  n_sel_total);
+        else if (per_cta <= 4 * 1024)
+            select_ratio_cluster_kernel<4><<<grid, 1024, 0, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                  n_sel_total);
+        else if (per_cta <= 8 * 1024)
+            select_ratio_cluster_kernel<8><<<grid, 1024, 0, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                  n_sel_total);
+        else
+            select_ratio_cluster_kernel<16><<<grid, 1024, 0, st>>>(gate_p, dims.B, dims.T, k, z, pos, cu_q, row_of,
+                                                                   n_sel_total);
         return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
     }
     if (ratio_mode) radix_select_kernel<<<dims.B, 1024, 0, st>>>(gate_p, dims.T, k, ws.th);

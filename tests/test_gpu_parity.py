@@ -84,7 +84,12 @@ SELECT_CASES = [
     ("normal", 4, 65536, 1, 0.0, 0.0625),
     ("ties", 3, 4097, 1, 0.0, 0.25),       # one-block ratio path: 16 tokens per thread, ragged
     ("ties", 2, 4096, 1, 0.0, 0.25),       # ... 4 tokens per thread, full
-    ("normal", 1, 16385, 1, 0.0, 0.125),   # just past the one-block path
+    ("normal", 1, 16385, 1, 0.0, 0.125),   # cluster path, 4 tokens per thread
+    ("normal", 2, 5000, 1, 0.0, 0.0),      # cluster path, k = 0
+    ("normal", 1, 9000, 1, 0.0, 1.0),      # cluster path, k = T
+    ("ties", 2, 32768, 1, 0.0, 0.5),       # cluster path, ties spanning every CTA
+    ("normal", 1, 131072, 1, 0.0, 0.125),  # largest cluster case, 16 tokens per thread
+    ("normal", 1, 140000, 1, 0.0, 0.01),   # beyond the cluster path: multi-launch radix select
 ]
 
 
