@@ -160,15 +160,15 @@ def make_device_inputs(w, device):
 
 
 CALLS = ["select", "local_fwd", "global_fwd", "combine", "combine_bwd", "global_bwd", "local_bwd"]
-LAUNCHES_PER_STEP = {"select": 4, "local_fwd": 1, "global_fwd": 3, "combine": 1, "combine_bwd": 1,
+LAUNCHES_PER_STEP = {"select": 4, "local_fwd": 1, "global_fwd": 4, "combine": 1, "combine_bwd": 1,
                      "global_bwd": 3, "local_bwd": 3}
 
 
 def launches_per_step(w):
     """Kernels one step launches: select takes one launch in ratio mode for
-    sequences of at most 16K tokens, four otherwise."""
+    sequences of at most 128K tokens, four otherwise."""
     n = sum(LAUNCHES_PER_STEP.values())
-    if w.mode == "ratio" and w.T <= 16384:
+    if w.mode == "ratio" and w.T <= 131072:
         n -= LAUNCHES_PER_STEP["select"] - 1
     return n
 

@@ -17,16 +17,28 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
 // One schedule entry of the global branch: a tile of up to 128 packed rows of
-// one sequence and the range of real positions it covers (App. B: the KV
-// blocks before min_pos need no causal predicate, those after max_pos none
-// at all).
+// one sequence, the range of real positions it covers (App. B: the KV blocks
+// before min_pos need no causal predicate, those after max_pos none at all),
+// and the KV blocks this entry visits: all of [0, max_pos / 128], or, when the
+// tiles are too few to fill the GPU, one share of that range whose partial
+// softmax result goes to a slot that a merge kernel combines with the others.
 struct GlobalTile {
     int row0;     // first packed row
     int nrows;    // rows in the tile (1..128)
     int b;        // sequence
     int min_pos;  // position of the first row
     int max_pos;  // position of the last row
+    int blk_lo;   // KV blocks visited (inclusive)
+    int blk_hi;
+    int slot;     // -1: the whole range, output written directly; else the partial-result slot
+    int cost;     // KV blocks visited (the ordering key)
     int pad0, pad1, pad2;
+};
+
+// A tile whose KV range is split: the merge kernel combines slots
+// slot0 .. slot0 + nsplit - 1 into its output rows.
+struct SplitTile {
+    int row0, nrows, slot0, nsplit;
 };
 
 // Everything the roles of a forward CTA need to know about one work item.
@@ -36,6 +48,7 @@ struct FwdItem {
     int nrows;      // valid rows
     int pos_min, pos_max;
     int blk_lo, blk_hi;  // inclusive KV block range
+    int slot;            // global split entry: partial-result slot; otherwise -1
 };
 
 // Does KV block n need the per-element visibility test for any row of the

@@ -63,6 +63,9 @@ struct FwdParams {
     const GlobalTile* tiles;       // global: schedule
     const int32_t* n_tiles;        // global: schedule length (device)
     int32_t* next_item;            // global: work counter, zeroed by the schedule kernel
+    float* o_part;                 // global split entries: unnormalised O [slot * Hq + h][D][128]
+    float* m_part;                 // ... their running max (log2 units) [slot * Hq + h][128]
+    float* l_part;                 // ... and their row sums
     int B, T, Hq, Hkv, window, cap;
     int q_tiles;                   // local: query tiles per sequence
     float scale_log2;              // softmax scale * log2(e)
@@ -84,6 +87,7 @@ __device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
         it.pos_max = it.row0 + it.nrows - 1;
         it.blk_lo = max(0, it.pos_min - p.window + 1) / kBN;
         it.blk_hi = it.pos_max / kBN;
+        it.slot = -1;
     } else {
         const GlobalTile g = p.tiles[tile];
         it.b = g.b;
@@ -91,8 +95,9 @@ __device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
         it.nrows = g.nrows;
         it.pos_min = g.min_pos;
         it.pos_max = g.max_pos;
-        it.blk_lo = 0;
-        it.blk_hi = g.max_pos / kBN;
+        it.blk_lo = g.blk_lo;
+        it.blk_hi = g.blk_hi;
+        it.slot = g.slot;
     }
     return it;
 }
@@ -444,6 +449,28 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
             __syncwarp();
             if (!ok) break;
             tc_fence_after();
+            if (GLOBAL && it.slot >= 0) {
+                // one share of a split KV range: unnormalised O, max and sum, for the
+                // merge.  O is stored transposed ([d][row]), so the warp's 32 rows
+                // of one column are one 128-byte line.
+                const int64_t unit = static_cast<int64_t>(it.slot) * p.Hq + it.h;
+                float* pcol = p.o_part + unit * kBM * D + r;
+                const uint32_t ocol = tmem + lane_off + C::kColO;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(ocol + c * 32, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) pcol[(c * 32 + i) * kBM] = __uint_as_float(v[i]);
+                }
+                tc_fence_before();
+                if (row_valid) {
+                    p.m_part[unit * kBM + r] = m_ref;
+                    p.l_part[unit * kBM + r] = l;
+                }
+                continue;
+            }
             const float inv_l = 1.0f / l;
             logo_bf16* orow;
             if (GLOBAL) orow = p.o + (static_cast<int64_t>(it.row0 + r) * p.Hq + it.h) * D;
@@ -483,17 +510,68 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
 }
 
 // ---------------------------------------------------------------- global prep
-// One block: split every sequence's packed rows into tiles of 128, and order
-// the tiles by their KV-block count, longest first.
+// Split-K of the global forward.  When the selected rows make too few work
+// items to fill the GPU (query tiles x heads < 2 x SMs: small sequences, high
+// sparsity), long tiles are cut into shares of their KV range, each share a
+// work item of its own that leaves its unnormalised O, row max and row sum in
+// a slot; merge_splits_kernel then combines the shares of each row exactly
+// (rescaling each share by 2^(m_s - M) to the common max M).  At most
+// kMaxPartialUnits (slot, head) pairs of partial results exist.
+constexpr int kMaxPartialUnits = 1024;
+constexpr int kMinSplitBlocks = 8;
+constexpr int kMaxShares = 64;  // shares of one tile
+// Splitting pays only when it shortens the longest item by more than the merge
+// and the extra items cost (measured: about a dozen blocks' time); below this
+// many blocks of gain the tiles stay whole.
+constexpr int kSplitMinGainBlocks = 24;
+
+// One block: split every sequence's packed rows into tiles of 128, split long
+// tiles' KV ranges if the tiles are too few, and order the entries by their
+// KV-block count, longest first.
+__device__ __forceinline__ int sched_block_scan(int v, int* total, int* sh)
+{
+    // exclusive scan over the 1024 threads, in thread order
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        const int w0 = sh[lane];
+        int w = w0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        sh[lane] = w - w0;
+        if (lane == 31) sh[32] = w;
+    }
+    __syncthreads();
+    const int r = sh[warp] + x - v;
+    *total = sh[32];
+    __syncthreads();
+    return r;
+}
+
 __global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __restrict__ pos,
-                                                               const int32_t* __restrict__ cu_q, int B,
-                                                               int32_t* __restrict__ tile_off,
+                                                               const int32_t* __restrict__ cu_q, int B, int Hq,
+                                                               int n_sm, int32_t* __restrict__ tile_off,
                                                                GlobalTile* __restrict__ unsorted,
                                                                GlobalTile* __restrict__ sorted,
                                                                int32_t* __restrict__ n_tiles,
-                                                               int32_t* __restrict__ next_item)
+                                                               int32_t* __restrict__ next_item,
+                                                               SplitTile* __restrict__ splits,
+                                                               int32_t* __restrict__ n_splits)
 {
-    __shared__ int sh_nt;
+    __shared__ int sh_nt, sh_chunk, sh_worth;
+    __shared__ int sh_scan[33];
+    __shared__ unsigned long long sh_total;
+    __shared__ int sh_longest;
     if (threadIdx.x == 0) {
         int acc = 0;
         for (int b = 0; b < B; ++b) {
@@ -502,12 +580,15 @@ __global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __
         }
         tile_off[B] = acc;
         sh_nt = acc;
-        *n_tiles = acc;
+        sh_total = 0;
+        sh_longest = 0;
         *next_item = 0;
     }
     __syncthreads();
     const int nt = sh_nt;
-    for (int t = threadIdx.x; t < nt; t += blockDim.x) {
+    // few tiles to fill the GPU with: split the long ones (then nt < 2 x SMs <= 1024)
+    const bool split = static_cast<int64_t>(nt) * Hq < 2ll * n_sm && Hq <= kMaxPartialUnits && nt <= 1024;
+    auto make_tile = [&](int t) {
         int lo = 0, hi = B - 1;
         while (lo < hi) {
             const int mid = (lo + hi + 1) >> 1;
@@ -521,19 +602,141 @@ __global__ void __launch_bounds__(1024) global_schedule_kernel(const int32_t* __
         g.b = b;
         g.min_pos = pos[g.row0];
         g.max_pos = pos[g.row0 + g.nrows - 1];
-        g.pad0 = g.max_pos / kBN + 1;  // cost: KV blocks visited
-        g.pad1 = g.pad2 = 0;
-        unsorted[t] = g;
+        g.blk_lo = 0;
+        g.blk_hi = g.max_pos / kBN;
+        g.slot = -1;
+        g.cost = g.blk_hi + 1;
+        g.pad0 = g.pad1 = g.pad2 = 0;
+        return g;
+    };
+    int ne = nt;
+    if (!split) {
+        for (int t = threadIdx.x; t < nt; t += blockDim.x) unsorted[t] = make_tile(t);
+        if (threadIdx.x == 0) *n_splits = 0;
+    } else {
+        // thread t < nt holds tile t
+        GlobalTile g{};
+        if (threadIdx.x < nt) {
+            g = make_tile(threadIdx.x);
+            atomicAdd(&sh_total, static_cast<unsigned long long>(g.cost));
+            atomicMax(&sh_longest, g.cost);
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            // cut only what is longer than an even share of the work per SM (the
+            // longest item bounds the launch; every extra item costs a pipeline
+            // restart and a partial write), in shares of at least kMinSplitBlocks
+            // blocks and at most kMaxShares per tile
+            const long long even = (static_cast<long long>(sh_total) * Hq + n_sm - 1) / n_sm;
+            int chunk = static_cast<int>(even > kMinSplitBlocks ? even : kMinSplitBlocks);
+            chunk = max(chunk, (sh_longest + kMaxShares - 1) / kMaxShares);
+            sh_chunk = chunk;
+            sh_worth = sh_longest - chunk >= kSplitMinGainBlocks;
+        }
+        __syncthreads();
     }
-    __syncthreads();
-    for (int t = threadIdx.x; t < nt; t += blockDim.x) {
-        const int c = unsorted[t].pad0;
+    if (split && !sh_worth) {  // too little to gain: the whole tiles after all
+        for (int t = threadIdx.x; t < nt; t += blockDim.x) unsorted[t] = make_tile(t);
+        if (threadIdx.x == 0) *n_splits = 0;
+    } else if (split) {
+        GlobalTile g{};
+        if (threadIdx.x < nt) g = make_tile(threadIdx.x);
+        // grow the shares until the split tiles fit in the partial-result slots
+        const int max_slots = kMaxPartialUnits / Hq;
+        int sp = 1, slots = 0;
+        for (;;) {
+            const int chunk = sh_chunk;
+            sp = threadIdx.x < nt ? (g.cost + chunk - 1) / chunk : 0;
+            sched_block_scan(sp > 1 ? sp : 0, &slots, sh_scan);
+            if (slots <= max_slots) break;
+            if (threadIdx.x == 0) sh_chunk = chunk * 2;
+            __syncthreads();
+        }
+        int n_entries, n_split_tiles;
+        const int e0 = sched_block_scan(threadIdx.x < nt ? sp : 0, &n_entries, sh_scan);
+        const int s0 = sched_block_scan(sp > 1 ? sp : 0, &slots, sh_scan);
+        const int t0 = sched_block_scan(sp > 1 ? 1 : 0, &n_split_tiles, sh_scan);
+        if (threadIdx.x < nt) {
+            if (sp == 1) {
+                unsorted[e0] = g;
+            } else {
+                splits[t0] = SplitTile{g.row0, g.nrows, s0, sp};
+                for (int s = 0; s < sp; ++s) {
+                    GlobalTile e = g;
+                    e.blk_lo = static_cast<int>(static_cast<int64_t>(g.cost) * s / sp);
+                    e.blk_hi = static_cast<int>(static_cast<int64_t>(g.cost) * (s + 1) / sp) - 1;
+                    e.slot = s0 + s;
+                    e.cost = e.blk_hi - e.blk_lo + 1;
+                    unsorted[e0 + s] = e;
+                }
+            }
+        }
+        if (threadIdx.x == 0) *n_splits = n_split_tiles;
+        ne = n_entries;
+    }
+    if (threadIdx.x == 0) *n_tiles = ne;
+    __syncthreads();  // entries written
+    for (int t = threadIdx.x; t < ne; t += blockDim.x) {
+        const int c = unsorted[t].cost;
         int rank = 0;
-        for (int u = 0; u < nt; ++u) {
-            const int cu = unsorted[u].pad0;
+        for (int u = 0; u < ne; ++u) {
+            const int cu = unsorted[u].cost;
             rank += (cu > c) || (cu == c && u < t);
         }
         sorted[rank] = unsorted[t];
+    }
+}
+
+// Combine the shares of every split tile: per (row, head), M = max_s m_s,
+// L = sum_s 2^(m_s - M) l_s, O = sum_s 2^(m_s - M) O_s / L, lse = (M + log2 L)
+// ln 2.  A share whose keys the row cannot see has m_s = -inf and weighs 0.
+// Work unit = (split tile, head, group of 8 columns); a block of 128 threads
+// (thread = row) takes units in a grid stride, so every unit's 8 x shares
+// loads per row are spread over the whole GPU; the transposed partials make
+// each of a warp's loads one 128-byte line.
+template <int D>
+__global__ void __launch_bounds__(128) merge_splits_kernel(const SplitTile* __restrict__ splits,
+                                                           const int32_t* __restrict__ n_splits, int Hq, int cap,
+                                                           const float* __restrict__ o_part,
+                                                           const float* __restrict__ m_part,
+                                                           const float* __restrict__ l_part,
+                                                           logo_bf16* __restrict__ o, float* __restrict__ lse)
+{
+    constexpr int kGroups = D / 8;
+    const int n_units = *n_splits * Hq * kGroups;
+    const int r = threadIdx.x;
+    for (int un = blockIdx.x; un < n_units; un += gridDim.x) {
+        const int g = un % kGroups, pr = un / kGroups;
+        const SplitTile st = splits[pr / Hq];
+        const int h = pr % Hq;
+        if (r >= st.nrows) continue;
+        const int64_t unit0 = static_cast<int64_t>(st.slot0) * Hq + h;  // share s: unit0 + s * Hq
+        float M = -INFINITY;
+        for (int s = 0; s < st.nsplit; ++s) M = fmaxf(M, m_part[(unit0 + static_cast<int64_t>(s) * Hq) * kBM + r]);
+        float L = 0.f;
+        float acc[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+        for (int s = 0; s < st.nsplit; ++s) {
+            const int64_t unit = unit0 + static_cast<int64_t>(s) * Hq;
+            const float m = m_part[unit * kBM + r];
+            const float w = m == -INFINITY ? 0.f : ex2_approx(m - M);
+            L += w * l_part[unit * kBM + r];
+            const float* src = o_part + unit * kBM * D + (g * 8) * kBM + r;
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = src[e * kBM];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[e] += w * v[e];
+        }
+        const float inv = 1.0f / L;
+        uint4 w4;
+        w4.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+        w4.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+        w4.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+        w4.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+        *reinterpret_cast<uint4*>(o + (static_cast<int64_t>(st.row0 + r) * Hq + h) * D + g * 8) = w4;
+        if (g == 0) lse[static_cast<int64_t>(h) * cap + st.row0 + r] = (M + log2f(L)) * kLn2;
     }
 }
 
@@ -544,23 +747,37 @@ struct GlobalFwdWs {
     int32_t* tile_off;
     int32_t* n_tiles;
     int32_t* next_item;
+    int32_t* n_splits;
+    SplitTile* splits;
+    float* o_part;
+    float* m_part;
+    float* l_part;
 };
 
 size_t global_fwd_ws_layout(const logo_dims& d, char* base, GlobalFwdWs* ws)
 {
     const size_t cap = static_cast<size_t>(d.B) * d.T;
     const size_t max_tiles = cap / kBM + d.B + 1;
+    const size_t max_entries = max_tiles + kMaxPartialUnits;  // each split adds at most one entry per slot
     size_t off = 0;
     const size_t o_qc = off;
     off = round_up(off + (cap + kBM) * d.Hq * d.D * 2, 256);
     const size_t o_un = off;
-    off = round_up(off + max_tiles * sizeof(GlobalTile), 256);
+    off = round_up(off + max_entries * sizeof(GlobalTile), 256);
     const size_t o_so = off;
-    off = round_up(off + max_tiles * sizeof(GlobalTile), 256);
+    off = round_up(off + max_entries * sizeof(GlobalTile), 256);
     const size_t o_to = off;
     off = round_up(off + (d.B + 1) * sizeof(int32_t), 256);
     const size_t o_nt = off;
-    off = round_up(off + 2 * sizeof(int32_t), 256);
+    off = round_up(off + 4 * sizeof(int32_t), 256);
+    const size_t o_sp = off;
+    off = round_up(off + max_tiles * sizeof(SplitTile), 256);
+    const size_t o_op = off;
+    off = round_up(off + static_cast<size_t>(kMaxPartialUnits) * kBM * d.D * sizeof(float), 256);
+    const size_t o_mp = off;
+    off = round_up(off + static_cast<size_t>(kMaxPartialUnits) * kBM * sizeof(float), 256);
+    const size_t o_lp = off;
+    off = round_up(off + static_cast<size_t>(kMaxPartialUnits) * kBM * sizeof(float), 256);
     if (ws) {
         ws->qc = reinterpret_cast<logo_bf16*>(base + o_qc);
         ws->unsorted = reinterpret_cast<GlobalTile*>(base + o_un);
@@ -568,6 +785,11 @@ size_t global_fwd_ws_layout(const logo_dims& d, char* base, GlobalFwdWs* ws)
         ws->tile_off = reinterpret_cast<int32_t*>(base + o_to);
         ws->n_tiles = reinterpret_cast<int32_t*>(base + o_nt);
         ws->next_item = ws->n_tiles + 1;
+        ws->n_splits = ws->n_tiles + 2;
+        ws->splits = reinterpret_cast<SplitTile*>(base + o_sp);
+        ws->o_part = reinterpret_cast<float*>(base + o_op);
+        ws->m_part = reinterpret_cast<float*>(base + o_mp);
+        ws->l_part = reinterpret_cast<float*>(base + o_lp);
     }
     return off;
 }
@@ -659,8 +881,9 @@ extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* 
     const int row_elems = dims.Hq * dims.D;
     const int gather_grid = max(1, min(cap + kBM, device_sm_count() * 8));
     gather_rows_kernel<<<gather_grid, 256, 0, st>>>(q, pos, cu_q, n_sel_total, dims.B, dims.T, row_elems, ws.qc);
-    global_schedule_kernel<<<1, 1024, 0, st>>>(pos, cu_q, dims.B, ws.tile_off, ws.unsorted, ws.sorted, ws.n_tiles,
-                                               ws.next_item);
+    const int n_sm = device_sm_count();
+    global_schedule_kernel<<<1, 1024, 0, st>>>(pos, cu_q, dims.B, dims.Hq, n_sm, ws.tile_off, ws.unsorted, ws.sorted,
+                                               ws.n_tiles, ws.next_item, ws.splits, ws.n_splits);
     if (cudaGetLastError() != cudaSuccess) return LOGO_ERR_CUDA;
     FwdParams prm{};
     if (!encode_bf16_4d(&prm.tm_q, ws.qc, dims.D, dims.Hq, static_cast<uint64_t>(cap) + kBM, 1, 64, kBM) ||
@@ -673,6 +896,9 @@ extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* 
     prm.tiles = ws.sorted;
     prm.n_tiles = ws.n_tiles;
     prm.next_item = ws.next_item;
+    prm.o_part = ws.o_part;
+    prm.m_part = ws.m_part;
+    prm.l_part = ws.l_part;
     prm.B = dims.B;
     prm.T = dims.T;
     prm.Hq = dims.Hq;
@@ -681,7 +907,17 @@ extern "C" int logo_global_sparse_attn_fwd(const logo_bf16* q, const logo_bf16* 
     prm.cap = cap;
     prm.q_tiles = 0;
     prm.scale_log2 = scale * kLog2e;
-    const int n_items_upper = static_cast<int>((static_cast<int64_t>(cap) / kBM + dims.B) * dims.Hq);
-    return dims.D == 128 ? launch_fwd<128, true>(prm, n_items_upper, st)
-                         : launch_fwd<64, true>(prm, n_items_upper, st);
+    const int n_items_upper =
+        static_cast<int>((static_cast<int64_t>(cap) / kBM + dims.B) * dims.Hq + kMaxPartialUnits);
+    rc = dims.D == 128 ? launch_fwd<128, true>(prm, n_items_upper, st) : launch_fwd<64, true>(prm, n_items_upper, st);
+    if (rc != LOGO_OK) return rc;
+    // always launched (a fixed launch sequence, capturable in a graph); exits at once without splits
+    const int merge_grid = n_sm * 4;
+    if (dims.D == 128)
+        merge_splits_kernel<128><<<merge_grid, 128, 0, st>>>(ws.splits, ws.n_splits, dims.Hq, cap, ws.o_part,
+                                                             ws.m_part, ws.l_part, o_c, lse_c);
+    else
+        merge_splits_kernel<64><<<merge_grid, 128, 0, st>>>(ws.splits, ws.n_splits, dims.Hq, cap, ws.o_part,
+                                                            ws.m_part, ws.l_part, o_c, lse_c);
+    return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }

@@ -36,9 +36,11 @@ def test_useful_flops_count_visible_pairs_only():
 
 
 def test_launch_count_per_step():
-    # 16K ratio workload: select 1, local fwd 1, global fwd 3 (gather, schedule,
-    # attention), combine 1, combine bwd 1, global bwd 3 (pre, attention, post),
-    # local bwd 3 (pre, attention, post)
-    assert bench.launches_per_step(WORKLOADS["16k"]) == 13
+    # 16K ratio workload: select 1, local fwd 1, global fwd 4 (gather, schedule,
+    # attention, merge of split KV ranges), combine 1, combine bwd 1, global bwd 3
+    # (pre, attention, post), local bwd 3 (pre, attention, post)
+    assert bench.launches_per_step(WORKLOADS["16k"]) == 14
+    # up to 128K tokens the selection is one cluster launch
+    assert bench.launches_per_step(WORKLOADS["64k"]) == 14
     # longer sequences take the four-launch selection
-    assert bench.launches_per_step(WORKLOADS["64k"]) == 16
+    assert bench.launches_per_step(WORKLOADS["64k"].with_(T=262144)) == 17
