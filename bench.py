@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "09669b4ffbb09292"): 826112512 + 479320832,
-    ("global_bwd", "09669b4ffbb09292"): 470733568 + 431303936,
+    ("local_bwd", "273d38505cd1baf4"): 824792832 + 479484928,
+    ("global_bwd", "273d38505cd1baf4"): 475473152 + 434990848,
 }
 
 
