@@ -140,3 +140,26 @@ def test_decode_step_fused_through_combine():
     ref_o, _, _ = oracle.combine_fwd(np32(o_l).reshape(B, 1, Hq, D), np32(o_c[:len(sel)]), p.numpy(), zc,
                                      row_of.cpu().numpy(), None, None, 1e-6)
     check_close(np32(o), ref_o, "step fused output")
+
+
+@pytest.mark.parametrize("D,Hq,Hkv", [(128, 4, 2), (64, 8, 2)])
+def test_decode_long_caches_many_chunks(D, Hq, Hkv):
+    """Few rows and long caches: each (row, KV head) is cut into many chunks
+    (for parallelism) whose partial results the last chunk to finish merges;
+    both the dense cache of the global call and a long ring of the local one."""
+    from paper_2608_29539_gb300 import logo as L
+    lens = [20000, 9000]
+    B, Lmax, W, R = len(lens), max(lens), 4096, 4096
+    kL, vL, kG, vG, qL, qG = _caches(B, Lmax, Hq, Hkv, D, seed=314 + D)
+    dev = torch.device("cuda")
+    seq_len = torch.tensor(lens, dtype=torch.int32, device=dev)
+    o_l = L.logo_decode_local_attn(qL.to(dev), _ring(kL, lens, R, W).to(dev), _ring(vL, lens, R, W).to(dev),
+                                   seq_len, W)
+    p = torch.full((B, 1), 0.9, dtype=torch.float32, device=dev)
+    z, pos, cu_q, row_of, n_sel = L.logo_select(p, L.LOGO_SELECT_THRESHOLD, b_th=0.5)
+    o_c = torch.zeros((B, Hq, D), dtype=torch.bfloat16, device=dev)
+    L.logo_decode_global_sparse_attn(qG.to(dev), _poisoned(kG, lens).to(dev), _poisoned(vG, lens).to(dev), seq_len,
+                                     cu_q, n_sel, o_c=o_c)
+    torch.cuda.synchronize()
+    check_close(np32(o_l), _oracle_new_token(qL, kL, vL, lens, W, [0, 1]), f"decode local long D{D}")
+    check_close(np32(o_c), _oracle_new_token(qG, kG, vG, lens, 0, [0, 1]), f"decode global long D{D}")
