@@ -51,6 +51,15 @@ struct FwdCfg {
     static constexpr uint32_t kColP0 = 384;  // P buffers (128 keys as bf16 pairs: 64 columns)
     static constexpr uint32_t kColP1 = 448;
     static constexpr uint32_t kTmemCols = 512;
+    // 12 warps: softmax (0..3), epilogue (4..7), producer / S issuer / P.V
+    // issuer (8..10, 11 idle).  Launched at 168 registers a thread (384 x 168 =
+    // 64,512); the softmax warpgroup takes 224 (its row of S lives in
+    // registers), the epilogue 168 (a row of O), the control warps 88:
+    // 128 x (224 + 168 + 88) = 61,440.
+    static constexpr int kThreads = 384;
+    static constexpr uint32_t kRegsSoftmax = 224;
+    static constexpr uint32_t kRegsEpilogue = 168;
+    static constexpr uint32_t kRegsControl = 88;
 };
 
 struct FwdParams {
@@ -103,14 +112,20 @@ __device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
 }
 
 template <int D, bool GLOBAL>
-__global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
+__global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
 {
     using C = FwdCfg<D>;
+    static_assert(128 * (C::kRegsSoftmax + C::kRegsEpilogue + C::kRegsControl) <= 384 * 168,
+                  "register split exceeds the launch allocation");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_drain, bar_drain_pv;
     __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_v_full[C::kStages], bar_kv_empty[C::kStages];
     __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2], bar_p_full[2], bar_p_free[2];
+    // softmax -> epilogue: 1/l of every row of an item (two slots), and O's
+    // columns free again once the epilogue has copied them out
+    __shared__ __align__(8) uint64_t bar_l_full[2], bar_l_empty[2], bar_o_free;
+    __shared__ float sh_inv_l[2][kBM];
     __shared__ uint32_t tmem_base_sh;
     __shared__ volatile int abort_flag;
     // global branch: items are taken dynamically (longest first, whichever CTA
@@ -137,17 +152,20 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
         }
         for (int s = 0; s < 4; ++s) {
             mbar_init(smem_u32(&bar_item_full[s]), 1);
-            mbar_init(smem_u32(&bar_item_empty[s]), 6);  // the two MMA threads + one lane per softmax warp
+            mbar_init(smem_u32(&bar_item_empty[s]), 10);  // the two MMA threads + one lane per softmax / epilogue warp
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_s_full[s]), 1);
             mbar_init(smem_u32(&bar_s_empty[s]), 128);
             mbar_init(smem_u32(&bar_p_full[s]), 128);
             mbar_init(smem_u32(&bar_p_free[s]), 1);
+            mbar_init(smem_u32(&bar_l_full[s]), 128);
+            mbar_init(smem_u32(&bar_l_empty[s]), 128);
         }
+        mbar_init(smem_u32(&bar_o_free), 128);
         fence_mbar_init();
     }
-    if (warp == 1) {
+    if (warp == 9) {
         tmem_alloc(smem_u32(&tmem_base_sh), C::kTmemCols);
         tmem_relinquish();
     }
@@ -177,7 +195,10 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
         return k;
     };
 
-    if (warp == 0) {
+    if (warp >= 8) {
+        // ------------------------------------------------------------ control warps
+        setmaxnreg_dec<C::kRegsControl>();
+    if (warp == 8) {
         // ------------------------------------------------------------ producer
         if (lane == 0) {
             tma_prefetch_desc(&p.tm_q);
@@ -236,7 +257,7 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
                     }
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == 9) {
         // ------------------------------------------------------------ S issuer
         // S = Q K^T of every block; the P.V products come from warp 6, so that
         // neither stream's waits leave the tensor pipe without queued work
@@ -279,7 +300,7 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
                 mbar_wait_drain(smem_u32(&bar_drain), 0);
             }
         }
-    } else if (warp == 6) {
+    } else if (warp == 10) {
         // ------------------------------------------------------------ P.V issuer
         if (lane == 0) {
             constexpr uint32_t idPV = idesc_bf16_f32(kBM, D, false, true);
@@ -293,10 +314,11 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
                 for (int j = 0; j < nblk && ok; ++j) {
                     const int itg = s_it + j;
                     const int st = (kv_it + j) % C::kStages, f = (kv_it + j) / C::kStages;
-                    // P of this block written (which also orders this P.V after the
-                    // previous item's epilogue: the softmax warps wrote P later)
                     if (!(ok = mbar_wait(smem_u32(&bar_p_full[itg & 1]), (itg >> 1) & 1, &abort_flag))) break;
                     if (!(ok = mbar_wait(smem_u32(&bar_v_full[st]), f & 1, &abort_flag))) break;
+                    // the item's first P.V overwrites O: the epilogue warps have
+                    // copied the previous item's O out of TMEM
+                    if (j == 0 && !(ok = mbar_wait(smem_u32(&bar_o_free), (item_i & 1) ^ 1, &abort_flag))) break;
                     tc_fence_after();
                     const uint32_t vbase = sV + st * C::kTileBytes;
                     const uint32_t pcol = tmem + ((itg & 1) ? C::kColP1 : C::kColP0);
@@ -317,8 +339,10 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
                 mbar_wait_drain(smem_u32(&bar_drain_pv), 0);
             }
         }
-    } else if (warp < 6) {
+    }
+    } else if (warp < 4) {
         // ------------------------------------------------------------ softmax
+        setmaxnreg_inc<C::kRegsSoftmax>();
         const int quad = warp & 3;  // TMEM lane quadrant this warp may access
         const int r = quad * 32 + lane;
         const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
@@ -444,66 +468,94 @@ __global__ void __launch_bounds__(224, 1) attn_fwd_kernel(const __grid_constant_
                 mbar_arrive(smem_u32(&bar_p_full[itg & 1]));
             }
             if (!ok) break;
-            // ---- epilogue: O / l, lse = (m + log2 l) * ln 2, once the last P.V is done
+            // ---- end of the item: lse = (m + log2 l) ln 2, and 1/l to the
+            //      epilogue warps, which normalise O while this warp moves on
+            if (row_valid) {
+                const float lse = (m_ref + log2f(l)) * kLn2;
+                if (GLOBAL && it.slot < 0) p.lse[static_cast<int64_t>(it.h) * p.cap + it.row0 + r] = lse;
+                else if (!GLOBAL) p.lse[(static_cast<int64_t>(it.b) * p.Hq + it.h) * p.T + it.row0 + r] = lse;
+            }
+            const int ls = item_i & 1;
+            ok = mbar_wait(smem_u32(&bar_l_empty[ls]), ((item_i >> 1) & 1) ^ 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            // a share of a split KV range hands over its row sum (the merge
+            // normalises); everything else 1/l
+            sh_inv_l[ls][r] = (GLOBAL && it.slot >= 0) ? l : 1.0f / l;
+            if (GLOBAL && it.slot >= 0 && row_valid)
+                p.m_part[(static_cast<int64_t>(it.slot) * p.Hq + it.h) * kBM + r] = m_ref;
+            mbar_arrive(smem_u32(&bar_l_full[ls]));
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        // warps 4..7: once an item's last P.V is done, copy O out of TMEM (then
+        // the next item's first P.V may overwrite it), and write O / l (or, for
+        // one share of a split KV range, the unnormalised O and the row sum)
+        setmaxnreg_dec<C::kRegsEpilogue>();
+        const int quad = warp & 3;
+        const int r = quad * 32 + lane;
+        const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+        int itg = 0;
+        bool ok = true;
+        for (int item_i = 0;; ++item_i) {
+            const int k = consume_item(item_i, &ok, true);
+            if (k < 0) break;
+            const FwdItem it = decode_item<GLOBAL>(p, k);
+            const bool row_valid = r < it.nrows;
+            itg += it.blk_hi - it.blk_lo + 1;
+            const int ls = item_i & 1;
+            ok = mbar_wait(smem_u32(&bar_l_full[ls]), (item_i >> 1) & 1, &abort_flag);
+            __syncwarp();
+            if (!ok) break;
+            const float lv = sh_inv_l[ls][r];
+            mbar_arrive(smem_u32(&bar_l_empty[ls]));
+            // the item's last P.V (block itg - 1) is done
             ok = mbar_wait(smem_u32(&bar_p_free[(itg - 1) & 1]), ((itg - 1) >> 1) & 1, &abort_flag);
             __syncwarp();
             if (!ok) break;
             tc_fence_after();
+            uint32_t ov[D / 32][32];
+            const uint32_t ocol = tmem + lane_off + C::kColO;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) tmem_ld32(ocol + c * 32, ov[c]);
+            tmem_wait_ld();
+            tc_fence_before();
+            mbar_arrive(smem_u32(&bar_o_free));
             if (GLOBAL && it.slot >= 0) {
-                // one share of a split KV range: unnormalised O, max and sum, for the
-                // merge.  O is stored transposed ([d][row]), so the warp's 32 rows
-                // of one column are one 128-byte line.
+                // one share of a split KV range: unnormalised O, stored transposed
+                // ([d][row]) so that the warp's 32 rows of a column are one line
                 const int64_t unit = static_cast<int64_t>(it.slot) * p.Hq + it.h;
                 float* pcol = p.o_part + unit * kBM * D + r;
-                const uint32_t ocol = tmem + lane_off + C::kColO;
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t v[32];
-                    tmem_ld32(ocol + c * 32, v);
-                    tmem_wait_ld();
+                for (int c = 0; c < D / 32; ++c)
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) pcol[(c * 32 + i) * kBM] = __uint_as_float(v[i]);
-                }
-                tc_fence_before();
-                if (row_valid) {
-                    p.m_part[unit * kBM + r] = m_ref;
-                    p.l_part[unit * kBM + r] = l;
-                }
+                    for (int i = 0; i < 32; ++i) pcol[(c * 32 + i) * kBM] = __uint_as_float(ov[c][i]);
+                if (row_valid) p.l_part[unit * kBM + r] = lv;
                 continue;
             }
-            const float inv_l = 1.0f / l;
+            if (!row_valid) continue;
+            const float inv_l = lv;
             logo_bf16* orow;
             if (GLOBAL) orow = p.o + (static_cast<int64_t>(it.row0 + r) * p.Hq + it.h) * D;
             else orow = p.o + ((static_cast<int64_t>(it.b) * p.T + it.row0 + r) * p.Hq + it.h) * D;
-            const uint32_t ocol = tmem + lane_off + C::kColO;
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(ocol + c * 32, v);
-                tmem_wait_ld();
-                if (row_valid) {
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(v[8 * q4 + 0]) * inv_l, __uint_as_float(v[8 * q4 + 1]) * inv_l);
-                        w.y = pack_bf16x2(__uint_as_float(v[8 * q4 + 2]) * inv_l, __uint_as_float(v[8 * q4 + 3]) * inv_l);
-                        w.z = pack_bf16x2(__uint_as_float(v[8 * q4 + 4]) * inv_l, __uint_as_float(v[8 * q4 + 5]) * inv_l);
-                        w.w = pack_bf16x2(__uint_as_float(v[8 * q4 + 6]) * inv_l, __uint_as_float(v[8 * q4 + 7]) * inv_l);
-                        *reinterpret_cast<uint4*>(orow + c * 32 + q4 * 8) = w;
-                    }
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const uint32_t* v = ov[c] + 8 * q4;
+                    uint4 w;
+                    w.x = pack_bf16x2(__uint_as_float(v[0]) * inv_l, __uint_as_float(v[1]) * inv_l);
+                    w.y = pack_bf16x2(__uint_as_float(v[2]) * inv_l, __uint_as_float(v[3]) * inv_l);
+                    w.z = pack_bf16x2(__uint_as_float(v[4]) * inv_l, __uint_as_float(v[5]) * inv_l);
+                    w.w = pack_bf16x2(__uint_as_float(v[6]) * inv_l, __uint_as_float(v[7]) * inv_l);
+                    *reinterpret_cast<uint4*>(orow + c * 32 + q4 * 8) = w;
                 }
-            }
-            tc_fence_before();
-            if (row_valid) {
-                const float lse = (m_ref + log2f(l)) * kLn2;
-                if (GLOBAL) p.lse[static_cast<int64_t>(it.h) * p.cap + it.row0 + r] = lse;
-                else p.lse[(static_cast<int64_t>(it.b) * p.Hq + it.h) * p.T + it.row0 + r] = lse;
             }
         }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 1) {
+    if (warp == 9) {
         tc_fence_after();
         tmem_dealloc(tmem, C::kTmemCols);
     }
@@ -804,7 +856,7 @@ int launch_fwd(const FwdParams& prm, int n_items_upper, cudaStream_t st)
         attr_done = true;
     }
     const int grid = max(1, min(n_items_upper, device_sm_count()));
-    attn_fwd_kernel<D, GLOBAL><<<grid, 224, C::kSmemBytes, st>>>(prm);
+    attn_fwd_kernel<D, GLOBAL><<<grid, C::kThreads, C::kSmemBytes, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 

@@ -168,6 +168,23 @@ __device__ __forceinline__ uint64_t policy_evict_first()
     return p;
 }
 
+// Move registers between warpgroups: every thread of a warpgroup executes one
+// of these with the same count (a multiple of 8), at the start of the code
+// that runs with that budget.  The sum over warpgroups of threads x count must
+// not exceed the block's threads x registers at launch, or an increase would
+// wait forever.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec()
+{
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc()
+{
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // ----------------------------------------------------------------- TMEM
 // Allocate `ncols` (power of two >= 32) TMEM columns; the base address is
 // written to shared memory at `dst_smem`.  Whole warp, .sync.aligned.
