@@ -363,6 +363,23 @@ def test_layer_step_4k_workload():
 
 
 # ------------------------------------------- full size, the benchmark's launch
+# Local backward shapes with several KV-block items per CTA on a 152-SM GPU
+# (each CTA walks 5-7 items): item sequences crossing sequences and KV
+# heads, GQA, a ragged last tile, a window of one.
+LOCAL_MANY_ITEM_CASES = [
+    # B, T, Hq, Hkv, D, W
+    (1, 8192, 16, 16, 128, 64),
+    (3, 5000, 16, 8, 128, 100),
+    (1, 12000, 8, 8, 128, 1),
+]
+
+
+@pytest.mark.parametrize("B,T,Hq,Hkv,D,W", LOCAL_MANY_ITEM_CASES)
+def test_local_bwd_many_items_per_cta(B, T, Hq, Hkv, D, W):
+    test_local_bwd(B, T, Hq, Hkv, D, W)
+    assert L().logo_get_device_status() == 0
+
+
 def test_full_size_16k_workload_sampled():
     """The headline 16K workload (B=1, H=32, d=128, T=16384, W=1024, clustered
     selection at ratio 1/8) through the same layer object bench.py times.
@@ -400,6 +417,10 @@ def test_full_size_16k_workload_sampled():
     check_close(np32(layer.dqL).reshape(-1, w.Hq, w.D)[:, h], rdq[:, h], "dqL head 7")
     check_close(np32(layer.dkL)[:, :, h], rdk[:, :, h], "dkL head 7")
     check_close(np32(layer.dvL)[:, :, h], rdv[:, :, h], "dvL head 7")
+    # dQ of every head on sampled rows
+    dO_l = np32(layer.dO_l).reshape(-1, w.Hq, w.D)
+    rdq, _, _ = oracle.attn_bwd(qL, kL, vL, np.zeros_like(rows), rows, w.window, dO_l[rows])
+    check_close(np32(layer.dqL).reshape(-1, w.Hq, w.D)[rows], rdq, "dqL sampled rows, every head")
     gb, gt = oracle.global_rows(opos, ocu)
     rdq, rdk, rdv = oracle.attn_bwd(qG, kG, vG, gb, gt, 0, np32(layer.dO_c)[:n], heads=h)
     dense = np.zeros((w.B, w.T, w.Hq, w.D))
