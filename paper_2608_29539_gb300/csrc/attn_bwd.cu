@@ -634,17 +634,14 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                     tc_fence_after();
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
                     const uint32_t scol = tmem + C::kColS;
+                    // S^T and dP^T k-steps alternate (two accumulators, both
+                    // needed before the softmax can start)
 #pragma unroll
                     for (int ks = 0; ks < D / 16; ++ks) {
                         const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;
                         const uint32_t kb = (ks >> 2) * 8192 + (ks & 3) * 32;
                         umma_bf16_ss(scol, sdesc_sw128(sK + ka, 16, 1024), sdesc_sw128(qb + kb, 16, 1024), idS,
                                      ks > 0 ? 1u : 0u);
-                    }
-#pragma unroll
-                    for (int ks = 0; ks < D / 16; ++ks) {
-                        const uint32_t ka = (ks >> 2) * 16384 + (ks & 3) * 32;
-                        const uint32_t kb = (ks >> 2) * 8192 + (ks & 3) * 32;
                         umma_bf16_ss(scol + 64, sdesc_sw128(sV + ka, 16, 1024), sdesc_sw128(ob + kb, 16, 1024), idS,
                                      ks > 0 ? 1u : 0u);
                     }
