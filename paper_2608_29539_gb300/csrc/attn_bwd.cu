@@ -670,9 +670,6 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                     const int b = u & 1, st = u % NS;
                     if (!(ok = mbar_wait(smem_u32(&bar_ds_full[b]), (u >> 1) & 1, &abort_flag))) break;
                     if (x == 0 && !(ok = mbar_wait(smem_u32(&bar_dkv_empty), (kv_items & 1) ^ 1, &abort_flag))) break;
-                    // dQ^T: the drain warps have read tile u-1's
-                    if (u > 0 && !(ok = mbar_wait(smem_u32(&bar_dq_empty[b ^ 1]), ((u - 1) >> 1) & 1, &abort_flag)))
-                        break;
                     tc_fence_after();
                     const uint32_t db = sDS + b * C::kPBytes;
                     const uint32_t qb = sQ + st * C::kQBytes, ob = sDO + st * C::kQBytes;
@@ -687,6 +684,11 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
                     // Q, dO of tile u are read: release the ring stage before dQ^T
                     // (which reads K and dS^T only), so the next load starts earlier
                     umma_commit(smem_u32(&bar_qdo_empty[st]));
+                    // dQ^T: the drain warps have read tile u-1's.  Waited for only
+                    // now, so that dV and dK never queue behind the drain.
+                    if (u > 0 && !(ok = mbar_wait(smem_u32(&bar_dq_empty[b ^ 1]), ((u - 1) >> 1) & 1, &abort_flag)))
+                        break;
+                    tc_fence_after();
 #pragma unroll
                     for (int ks = 0; ks < kBN / 16; ++ks) {
                         umma_bf16_ss(tmem + C::kColDQ, sdesc_sw128(sK + ks * 2048, 16384, 1024),
