@@ -3,28 +3,34 @@
 //   logo_local_attn_fwd          O^L = SoftmaxAttn_W(Q^L, K^L, V^L)   (Eq. 6)
 //   logo_global_sparse_attn_fwd  O^G_I = SoftmaxAttn_inf(Q^G_I, K^G, V^G) (Eq. 8)
 //
-// One persistent kernel template serves both.  A CTA (7 warps) loops over
+// One persistent kernel template serves both.  A CTA (12 warps) loops over
 // work items = (128-row query tile, query head):
-//   warp 0      TMA producer: Q tile once per item, then K/V blocks through a
-//               ring of shared-memory stages (128-byte swizzle).
-//   warp 1      S issuer (one thread): S = Q K^T into one of two TMEM S buffers.
-//   warp 6      P.V issuer (one thread): O += P V into the TMEM O accumulator
+//   warp 8      TMA producer: Q tile once per item, then K blocks (local: K
+//               and V blocks) through a ring of shared-memory stages
+//               (128-byte swizzle)
+//   warp 11     global branch: V blocks through a ring of their own
+//   warp 9      S issuer (one thread): S = Q K^T into one of two TMEM S buffers
+//   warp 10     P.V issuer (one thread): O += P V into the TMEM O accumulator
 //               with P read straight from TMEM.  Two issuing threads keep the
 //               tensor pipe fed while either waits for its inputs: the issue
 //               queue is short, so a single thread that stops to wait starves
 //               the pipe (measured: 1728 vs 2427 TFLOP/s on the same MMA stream).
-//   warps 2..5  softmax: one thread per query row (its TMEM lane).  Online
+//   warps 0..3  softmax: one thread per query row (its TMEM lane).  Online
 //               softmax in the log2 domain with conditional rescaling of O
 //               (only when the running max grows by more than 2^8); P goes
 //               back to TMEM as bf16 pairs, into one of two P buffers, so the
 //               softmax of block n never waits for the P.V of block n-1
 //               unless it has to rescale O.
+//   warps 4..7  epilogue: O out of TMEM once an item's last P.V is done,
+//               normalised and stored while the softmax warps start the next
+//               item.
 // The KV blocks of an item are only those some row can see; blocks where
 // every row sees every key skip the per-element predicate (App. B's
 // three-region traversal; for the local branch the window edge is a second
-// masked region).  Global items come from a schedule ordered by cost
-// (longest first) that a one-block kernel builds on the device, so nothing
-// here needs the selected count on the host.
+// masked region), and inside a masked block only the 32-key groups a row
+// sees in part are tested key by key.  Global items come from a schedule
+// ordered by cost (longest first) that a one-block kernel builds on the
+// device, so nothing here needs the selected count on the host.
 #include <cuda_bf16.h>
 
 #include <cstdint>
@@ -40,7 +46,13 @@ template <int D>
 struct FwdCfg {
     static constexpr int kSub = D / 64;             // 64-column (128-byte) sub-tiles per row
     static constexpr int kTileBytes = kBM * D * 2;  // one Q / K / V tile
-    static constexpr int kStages = 3;               // K/V ring depth
+    // K/V ring of three stages.  The global branch runs K and V as two rings
+    // with a producer each: a K stage is free once S of its block is done, a
+    // V stage once P.V is, so K loads run further ahead (global fwd -7% at
+    // 16K).  The local branch keeps one producer loading K and V of a block
+    // together into one stage that P.V frees (its short items ran 6% slower
+    // with the split).
+    static constexpr int kStages = 3;
     static constexpr int kOffQ = 0;
     static constexpr int kOffK = kOffQ + kTileBytes;
     static constexpr int kOffV = kOffK + kStages * kTileBytes;
@@ -51,8 +63,8 @@ struct FwdCfg {
     static constexpr uint32_t kColP0 = 384;  // P buffers (128 keys as bf16 pairs: 64 columns)
     static constexpr uint32_t kColP1 = 448;
     static constexpr uint32_t kTmemCols = 512;
-    // 12 warps: softmax (0..3), epilogue (4..7), producer / S issuer / P.V
-    // issuer (8..10, 11 idle).  Launched at 168 registers a thread (384 x 168 =
+    // 12 warps: softmax (0..3), epilogue (4..7), Q/K(/V) producer, S issuer,
+    // P.V issuer, global branch: V producer (8..11).  Launched at 168 registers a thread (384 x 168 =
     // 64,512); the softmax warpgroup takes 224 (its row of S lives in
     // registers), the epilogue 168 (a row of O), the control warps 88:
     // 128 x (224 + 168 + 88) = 61,440.
@@ -111,6 +123,47 @@ __device__ __forceinline__ FwdItem decode_item(const FwdParams& p, int k)
     return it;
 }
 
+// Visibility inside one 128-key block: the row sees keys c with lo <= c <= hi;
+// every other s[c] becomes -inf.  Called by all 32 lanes of a warp, whose rows
+// are consecutive, so most 32-key groups are seen whole by every row of the
+// warp or by none of them; one warp reduction classifies the groups.  Selects
+// and moves cost two issue cycles per warp on this pipe, so only the groups
+// in between get the per-key select, and only against the bound that cuts
+// them; unseen groups get plain moves.
+__device__ __forceinline__ void mask_row_block(float (&s)[kBN], int lo, int hi)
+{
+    uint32_t cls = 0;  // per group g: bit g seen whole, 4+g unseen, 8+g lo does not cut, 12+g hi does not cut
+#pragma unroll
+    for (int g = 0; g < kBN / 32; ++g) {
+        const bool lo_cuts = lo > 32 * g, hi_cuts = hi < 32 * g + 31;
+        cls |= (!lo_cuts && !hi_cuts) ? (1u << g) : 0u;
+        cls |= (hi < 32 * g || lo > 32 * g + 31) ? (16u << g) : 0u;
+        cls |= lo_cuts ? 0u : (256u << g);
+        cls |= hi_cuts ? 0u : (4096u << g);
+    }
+    cls = __reduce_and_sync(0xffffffffu, cls);
+#pragma unroll
+    for (int g = 0; g < kBN / 32; ++g) {
+        if (cls & (1u << g)) continue;
+        if (cls & (16u << g)) {
+            // (an opaque move: a constant assigned in this branch made the
+            // compiler spill the row)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) asm volatile("mov.b32 %0, 0xff800000;" : "=f"(s[32 * g + i]));
+        } else if (cls & (256u << g)) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s[32 * g + i] = 32 * g + i <= hi ? s[32 * g + i] : -INFINITY;
+        } else if (cls & (4096u << g)) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s[32 * g + i] = 32 * g + i >= lo ? s[32 * g + i] : -INFINITY;
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                s[32 * g + i] = (32 * g + i >= lo && 32 * g + i <= hi) ? s[32 * g + i] : -INFINITY;
+        }
+    }
+}
+
 template <int D, bool GLOBAL>
 __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant__ FwdParams p)
 {
@@ -120,7 +173,10 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t bar_q_full, bar_q_empty, bar_drain, bar_drain_pv;
-    __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_v_full[C::kStages], bar_kv_empty[C::kStages];
+    // bar_k_empty frees a K stage (global) or a K/V stage (local); bar_v_empty
+    // a V stage (global only)
+    __shared__ __align__(8) uint64_t bar_k_full[C::kStages], bar_k_empty[C::kStages];
+    __shared__ __align__(8) uint64_t bar_v_full[C::kStages], bar_v_empty[C::kStages];
     __shared__ __align__(8) uint64_t bar_s_full[2], bar_s_empty[2], bar_p_full[2], bar_p_free[2];
     // softmax -> epilogue: 1/l of every row of an item (two slots), and O's
     // columns free again once the epilogue has copied them out
@@ -147,12 +203,14 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
         mbar_init(smem_u32(&bar_drain_pv), 1);
         for (int s = 0; s < C::kStages; ++s) {
             mbar_init(smem_u32(&bar_k_full[s]), 1);
+            mbar_init(smem_u32(&bar_k_empty[s]), 1);
             mbar_init(smem_u32(&bar_v_full[s]), 1);
-            mbar_init(smem_u32(&bar_kv_empty[s]), 1);
+            mbar_init(smem_u32(&bar_v_empty[s]), 1);
         }
         for (int s = 0; s < 4; ++s) {
             mbar_init(smem_u32(&bar_item_full[s]), 1);
-            mbar_init(smem_u32(&bar_item_empty[s]), 10);  // the two MMA threads + one lane per softmax / epilogue warp
+            // the V producer, the two MMA threads, one lane per softmax / epilogue warp
+            mbar_init(smem_u32(&bar_item_empty[s]), 11);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(smem_u32(&bar_s_full[s]), 1);
@@ -234,16 +292,19 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                 ++q_fills;
                 for (int n = it.blk_lo; n <= it.blk_hi; ++n, ++kv_it) {
                     const int st = kv_it % C::kStages, f = kv_it / C::kStages;
-                    if (!(ok = mbar_wait(smem_u32(&bar_kv_empty[st]), (f & 1) ^ 1, &abort_flag))) break;
-                    const uint32_t kb = smem_u32(&bar_k_full[st]), vb = smem_u32(&bar_v_full[st]);
+                    if (!(ok = mbar_wait(smem_u32(&bar_k_empty[st]), (f & 1) ^ 1, &abort_flag))) break;
+                    const uint32_t kb = smem_u32(&bar_k_full[st]);
                     mbar_arrive_expect_tx(kb, C::kTileBytes);
                     for (int s = 0; s < C::kSub; ++s)
                         tma_load_4d(sK + st * C::kTileBytes + s * 16384, &p.tm_k, kb, 64 * s, it.kvh, n * kBN, it.b,
                                     pol_kv);
-                    mbar_arrive_expect_tx(vb, C::kTileBytes);
-                    for (int s = 0; s < C::kSub; ++s)
-                        tma_load_4d(sV + st * C::kTileBytes + s * 16384, &p.tm_v, vb, 64 * s, it.kvh, n * kBN, it.b,
-                                    pol_kv);
+                    if (!GLOBAL) {  // V of the same block into the same stage
+                        const uint32_t vb = smem_u32(&bar_v_full[st]);
+                        mbar_arrive_expect_tx(vb, C::kTileBytes);
+                        for (int s = 0; s < C::kSub; ++s)
+                            tma_load_4d(sV + st * C::kTileBytes + s * 16384, &p.tm_v, vb, 64 * s, it.kvh, n * kBN,
+                                        it.b, pol_kv);
+                    }
                     last_fill[st] = f;
                 }
                 if (!ok) break;
@@ -253,7 +314,7 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                 for (int s = 0; s < C::kStages; ++s)
                     if (last_fill[s] >= 0) {
                         mbar_wait_drain(smem_u32(&bar_k_full[s]), last_fill[s] & 1);
-                        mbar_wait_drain(smem_u32(&bar_v_full[s]), last_fill[s] & 1);
+                        if (!GLOBAL) mbar_wait_drain(smem_u32(&bar_v_full[s]), last_fill[s] & 1);
                     }
             }
         }
@@ -289,6 +350,7 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                                      ks > 0 ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_s_full[buf]));
+                    if (GLOBAL) umma_commit(smem_u32(&bar_k_empty[st]));  // K of this block is read
                 }
                 if (!ok) break;
                 umma_commit(smem_u32(&bar_q_empty));
@@ -328,7 +390,8 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                         umma_bf16_ts(tmem + C::kColO, pcol + ks * 8, bdesc, idPV, (j > 0 || ks > 0) ? 1u : 0u);
                     }
                     umma_commit(smem_u32(&bar_p_free[itg & 1]));
-                    umma_commit(smem_u32(&bar_kv_empty[st]));  // K was read by S of this block, done before P
+                    // V of this block is read (local: K and V, whose S was done before P)
+                    umma_commit(smem_u32(GLOBAL ? &bar_v_empty[st] : &bar_k_empty[st]));
                 }
                 if (!ok) break;
                 kv_it += nblk;
@@ -337,6 +400,37 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
             if (!ok) {
                 umma_commit(smem_u32(&bar_drain_pv));
                 mbar_wait_drain(smem_u32(&bar_drain_pv), 0);
+            }
+        }
+    } else if (GLOBAL && warp == 11) {
+        // ------------------------------------------------------------ V producer
+        // global branch: V blocks through their own ring (a stage is freed by
+        // the P.V that read it), so a V load never holds up the next K load
+        if (lane == 0) {
+            const uint64_t pol_kv = policy_evict_last();
+            int kv_it = 0;
+            int last_fill[C::kStages];
+            for (int s = 0; s < C::kStages; ++s) last_fill[s] = -1;
+            bool ok = true;
+            for (int item_i = 0;; ++item_i) {
+                const int k = consume_item(item_i, &ok, false);
+                if (k < 0) break;
+                const FwdItem it = decode_item<GLOBAL>(p, k);
+                for (int n = it.blk_lo; n <= it.blk_hi; ++n, ++kv_it) {
+                    const int st = kv_it % C::kStages, f = kv_it / C::kStages;
+                    if (!(ok = mbar_wait(smem_u32(&bar_v_empty[st]), (f & 1) ^ 1, &abort_flag))) break;
+                    const uint32_t vb = smem_u32(&bar_v_full[st]);
+                    mbar_arrive_expect_tx(vb, C::kTileBytes);
+                    for (int s = 0; s < C::kSub; ++s)
+                        tma_load_4d(sV + st * C::kTileBytes + s * 16384, &p.tm_v, vb, 64 * s, it.kvh, n * kBN, it.b,
+                                    pol_kv);
+                    last_fill[st] = f;
+                }
+                if (!ok) break;
+            }
+            if (!ok) {  // let copies already issued land before the CTA exits
+                for (int s = 0; s < C::kStages; ++s)
+                    if (last_fill[s] >= 0) mbar_wait_drain(smem_u32(&bar_v_full[s]), last_fill[s] & 1);
             }
         }
     }
@@ -379,11 +473,8 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                 }
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_s_empty[buf]));
-                if (block_needs_mask(n, it.pos_min, it.pos_max, window)) {
-#pragma unroll
-                    for (int c = 0; c < kBN; ++c)
-                        if (!key_visible(n * kBN + c, mypos, window)) s[c] = -INFINITY;
-                }
+                if (block_needs_mask(n, it.pos_min, it.pos_max, window))
+                    mask_row_block(s, mypos - window + 1 - n * kBN, mypos - n * kBN);
                 // 4 independent 3-input max chains and 4 packed-pair sums keep
                 // dependency chains short; exp arguments are formed two at a
                 // time with f32x2 FMAs
