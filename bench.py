@@ -45,8 +45,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "273d38505cd1baf4"): 824792832 + 479484928,
-    ("global_bwd", "273d38505cd1baf4"): 475473152 + 434990848,
+    ("local_bwd", "719cf024947d3e17"): 824331776 + 479615232,
+    ("global_bwd", "719cf024947d3e17"): 470104320 + 431910400,
 }
 
 
