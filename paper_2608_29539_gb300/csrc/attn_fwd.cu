@@ -453,11 +453,18 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
             else mypos = row_valid ? it.row0 + r : it.pos_max;
             float m_ref = -INFINITY;  // running max, log2 domain
             float l = 0.f;
+            // The S-ready and P-buffer-free barriers are nearly always complete
+            // by the time they are needed; each is tested (non-blocking) well
+            // before that point, so the test's latency overlaps other work, and
+            // only a warp that found one incomplete waits on it.
+            bool s_ready = false;  // S of this block seen complete while the previous block ended
             for (int n = it.blk_lo; n <= it.blk_hi; ++n, ++itg) {
                 const int buf = itg & 1, use = itg >> 1;
-                ok = mbar_wait(smem_u32(&bar_s_full[buf]), use & 1, &abort_flag);
-                __syncwarp();
-                if (!ok) break;
+                if (!s_ready) {
+                    ok = mbar_wait(smem_u32(&bar_s_full[buf]), use & 1, &abort_flag);
+                    __syncwarp();
+                    if (!ok) break;
+                }
                 tc_fence_after();
                 float s[kBN];
                 const uint32_t scol = tmem + lane_off + (buf ? C::kColS1 : C::kColS0);
@@ -473,6 +480,8 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                 }
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_s_empty[buf]));
+                // P buffer itg%2 is free once the P.V two blocks back is done
+                const bool p_free_seen = mbar_test(smem_u32(&bar_p_free[itg & 1]), ((itg >> 1) & 1) ^ 1);
                 if (block_needs_mask(n, it.pos_min, it.pos_max, window))
                     mask_row_block(s, mypos - window + 1 - n * kBN, mypos - n * kBN);
                 // 4 independent 3-input max chains and 4 packed-pair sums keep
@@ -541,10 +550,11 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                         tmem_st32(ocol + c * 32, v);
                     }
                 }
-                // P buffer itg%2 is free once the P.V two blocks back is done
-                ok = mbar_wait(smem_u32(&bar_p_free[itg & 1]), ((itg >> 1) & 1) ^ 1, &abort_flag);
-                __syncwarp();
-                if (!ok) break;
+                if (!__all_sync(0xffffffffu, p_free_seen)) {
+                    ok = mbar_wait(smem_u32(&bar_p_free[itg & 1]), ((itg >> 1) & 1) ^ 1, &abort_flag);
+                    __syncwarp();
+                    if (!ok) break;
+                }
                 tc_fence_after();
                 const uint32_t pcol = tmem + lane_off + ((itg & 1) ? C::kColP1 : C::kColP0);
 #pragma unroll
@@ -554,9 +564,11 @@ __global__ void __launch_bounds__(384, 1) attn_fwd_kernel(const __grid_constant_
                     for (int i = 0; i < 32; ++i) pk[i] = cvt_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
                     tmem_st32(pcol + 32 * h, pk);
                 }
+                const bool s_seen = n < it.blk_hi && mbar_test(smem_u32(&bar_s_full[(itg + 1) & 1]), ((itg + 1) >> 1) & 1);
                 tmem_wait_st();
                 tc_fence_before();
                 mbar_arrive(smem_u32(&bar_p_full[itg & 1]));
+                s_ready = __all_sync(0xffffffffu, s_seen);
             }
             if (!ok) break;
             // ---- end of the item: lse = (m + log2 l) ln 2, and 1/l to the

@@ -82,6 +82,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity (acquire, CTA scope).
+// Issued well before its result is needed, its latency overlaps other work;
+// a caller that finds the phase not yet complete falls back to mbar_wait.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred P;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 P, [%1], %2;\n\t"
+        "selp.b32 %0, 1, 0, P;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Wall-clock budget of one wait: far above any legitimate wait in these
 // kernels (a whole launch takes milliseconds), far below a watchdog.
 constexpr uint64_t kWaitBudgetNs = 2000000000ull;
