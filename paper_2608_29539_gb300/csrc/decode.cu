@@ -10,13 +10,17 @@
 //                                   sequence's whole dense cache (Eq. 8)
 //
 // Both run one persistent kernel per call.  An item is one chunk of cache
-// rows (up to kDecSubMax sub-tiles of 128 rows) of one (row, KV head); a CTA
+// rows (up to kDecSubMax sub-tiles of 64 rows) of one (row, KV head); a CTA
 // (4 warps) walks its items' sub-tiles through a 3-stage TMA ring (128-byte
-// swizzle), so the next two sub-tiles load while one is computed, and serves
-// every query head of the KV head's group from each: S = q.K^T and O = P.V as
-// warp-level bf16 products (mma.sync m16n8k16: the group's heads are the 16
-// rows, so a group of up to 16 heads fills one tile), with an online softmax
-// (running max and sum per head, in log2 units) across the item's sub-tiles.
+// swizzle), a stage refilled once all four warps have released it, and
+// serves every query head of the KV head's group from each: S = q.K^T and
+// O = P.V as warp-level bf16 products (mma.sync m16n8k16: the group's heads
+// are the 16 rows, so a group of up to 16 heads fills one tile).  Each warp
+// takes 16 rows of every sub-tile and keeps its own online softmax (running
+// max and sum per head, in log2 units) across the item's sub-tiles, P going
+// from the S fragments straight into the A fragments of the P.V product, so
+// nothing inside the sub-tile loop waits for another warp; the four warps'
+// results are combined exactly at the end of the item.
 // A row whose cache fits one chunk gets its output written by that item.
 // Longer caches are split into chunks for parallelism: each chunk leaves its
 // unnormalised O, max and sum, and the last chunk of a (row, KV head) to
@@ -64,11 +68,11 @@ struct DecCfg {
     static constexpr int kHalfBytes = kDecRows * 128;         // 64 head-dim columns of the sub-tile's rows
     static constexpr int kTileBytes = (D / 64) * kHalfBytes;  // K or V sub-tile
     static constexpr int kStageBytes = 2 * kTileBytes;        // K then V
-    static constexpr int kOffS = kDecStages * kStageBytes;    // [group][rows] fp32 scores, then P
-    static constexpr int kSmemBytes = kOffS + kDecMaxGroup * kDecRows * 4 + 1024;
-    // the warps' partial O at the end of an item go to the stage consumed last
-    // (no copy targets it before the next item's first issue)
-    static_assert(4 * kDecMaxGroup * D * 4 <= kStageBytes, "partial O of four warps must fit in a stage");
+    static constexpr int kOffW = kDecStages * kStageBytes;    // chunk-merge weights [group][chunks] fp32
+    static constexpr int kOffM = kOffW + 16 * 64 * 4;         // the warps' partial results, sized per group:
+    // [warp][group][D + 2] fp32: unnormalised o, then m, l
+    static constexpr int merge_bytes(int group) { return 4 * group * (D + 2) * 4; }
+    static constexpr int smem_bytes(int group) { return kOffM + merge_bytes(group) + 1024; }
 };
 constexpr int kDecMaxChunks = 64;  // chunks per cache at most (the merge's weights: group x chunks <= 16 x 64)
 
@@ -113,28 +117,35 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
     using C = DecCfg<D>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t bar_full[kDecStages];
+    // bar_full: a stage's K/V sub-tile landed; bar_empty: the four warps are done with it
+    __shared__ __align__(8) uint64_t bar_full[kDecStages], bar_empty[kDecStages];
     __shared__ volatile int abort_flag;
-    __shared__ float sh_m[kDecMaxGroup], sh_l[kDecMaxGroup], sh_alpha[kDecMaxGroup];
     __shared__ int sh_last;
+    __shared__ float sh_wm[4][kDecMaxGroup];  // per head: weight of each warp's partial, 1 / L
+    __shared__ float sh_M[kDecMaxGroup], sh_L[kDecMaxGroup];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int gid = lane >> 2, tig = lane & 3;  // mma fragment coordinates
     const int mi = lane >> 3, rr = lane & 7;    // ldmatrix: matrix index, row in the matrix
     const int group = p.Hq / p.Hkv;
-    float* sS = reinterpret_cast<float*>(smem + C::kOffS);
+    float* sW = reinterpret_cast<float*>(smem + C::kOffW);
+    float* sM = reinterpret_cast<float*>(smem + C::kOffM);
     const uint32_t sRing = smem_u32(smem);
     // rows of the call: every sequence (local), the selected packed rows (global)
     const int n_rows = RING ? p.B : *p.n_sel;
     const long long n_items = static_cast<long long>(n_rows) * p.Hkv * p.nchunk;
     if (tid == 0) {
         abort_flag = 0;
-        for (int s = 0; s < kDecStages; ++s) mbar_init(smem_u32(&bar_full[s]), 1);
+        for (int s = 0; s < kDecStages; ++s) {
+            mbar_init(smem_u32(&bar_full[s]), 1);
+            mbar_init(smem_u32(&bar_empty[s]), 4);
+        }
         fence_mbar_init();
     }
     __syncthreads();
 
     // ---- the producer (thread 0) walks the same sequence of sub-tiles as the
-    //      consumers, kDecStages - 1 ahead: (item w, sub-tile s) in order
+    //      consumers, up to kDecStages ahead: (item w, sub-tile s) in order; a
+    //      stage is refilled once every warp has released it
     long long pw = blockIdx.x;
     int ps = 0, ps1 = 0;
     auto producer_next = [&](DecItem* it_out) -> bool {  // the next sub-tile to load, or false
@@ -150,10 +161,12 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
     };
     DecItem pit{};
     int issued = 0;
+    bool ok = true;
     auto issue = [&]() {
-        if (tid != 0) return;
+        if (tid != 0 || !ok) return;
         if (!producer_next(&pit)) return;
         const int st = issued % kDecStages;
+        if (!(ok = mbar_wait(smem_u32(&bar_empty[st]), ((issued / kDecStages) & 1) ^ 1, &abort_flag))) return;
         const uint32_t bar = smem_u32(&bar_full[st]);
         const uint32_t base = sRing + st * C::kStageBytes;
         const uint64_t pol = policy_evict_first();
@@ -168,8 +181,14 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
     };
     for (int i = 0; i < kDecStages - 1; ++i) issue();
 
+    // Each warp takes 16 rows of every sub-tile (rows 16w..16w+15) and keeps an
+    // online softmax of its own across the item's sub-tiles, so no instruction
+    // inside the sub-tile loop waits for another warp: S = q.K^T lands in mma
+    // fragments, P = 2^(S - m) goes from those straight into the A fragments
+    // of O += P.V (a pair of 8-column S tiles is one 16-deep A fragment), and
+    // the four warps' results are combined once per item.
+    constexpr int NT = D / 8;
     int consumed = 0;
-    bool ok = true;
     for (long long w = blockIdx.x; w < n_items && ok; w += gridDim.x) {
         const DecItem it = dec_item<RING>(p, w);
         if (it.s0 >= it.s1) continue;
@@ -188,11 +207,9 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
                 }
             }
         }
-        if (tid < kDecMaxGroup) {
-            sh_m[tid] = -INFINITY;
-            sh_l[tid] = 0.f;
-        }
-        constexpr int NT = D / 8;
+        // this lane's two heads (fragment rows gid and gid + 8): running max
+        // (log2 units), running sum, and O
+        float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
         float oc[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
@@ -200,143 +217,150 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
             for (int i = 0; i < 4; ++i) oc[nt][i] = 0.f;
 
         for (int s = it.s0; s < it.s1; ++s, ++consumed) {
-            issue();  // the stage freed by the sub-tile before this one
+            issue();
             const int st = consumed % kDecStages;
             const uint32_t sK = sRing + st * C::kStageBytes, sV = sK + C::kTileBytes;
-            if (!(ok = mbar_wait(smem_u32(&bar_full[st]), (consumed / kDecStages) & 1, &abort_flag))) break;
-            const int j0 = s * kDecRows;
-            if (tid < kDecRows) {
+            ok = mbar_wait(smem_u32(&bar_full[st]), (consumed / kDecStages) & 1, &abort_flag) && ok;
+            if (!(ok = __all_sync(0xffffffffu, ok))) break;  // the warp leaves together (mma.sync needs all lanes)
+            const int j0 = s * kDecRows + warp * kDecRowsPerWarp;  // this warp's first cache row
+            if (lane < kDecRowsPerWarp) {
                 // a cache row the token does not see may hold anything, NaN included:
                 // zero its V so that P = 0 keeps it out of the product
-                const int spos = pos_of<RING>(j0 + tid, it.len, p.R);
+                const int spos = pos_of<RING>(j0 + lane, it.len, p.R);
                 const bool vis = spos >= 0 && (!RING || spos > it.len - 1 - p.window);
                 if (!vis) {
+                    const int row = warp * kDecRowsPerWarp + lane;
 #pragma unroll
                     for (int half = 0; half < D / 64; ++half)
 #pragma unroll
                         for (int ch = 0; ch < 8; ++ch)
-                            st_shared_v4(sV + half * C::kHalfBytes + sw128_offset(tid, ch), 0u, 0u, 0u, 0u);
+                            st_shared_v4(sV + half * C::kHalfBytes + sw128_offset(row, ch), 0u, 0u, 0u, 0u);
                 }
             }
-            // ---- S = q.K^T: warp w takes cache rows [16w, 16w + 16) (two 8-row tiles)
-            {
-                constexpr int NTW = kDecRowsPerWarp / 8;
-                float sc[NTW][4];
+            __syncwarp();
+            // ---- S = q.K^T over the warp's 16 rows (two 8-row tiles)
+            float sc[2][4];
 #pragma unroll
-                for (int nt = 0; nt < NTW; ++nt)
+            for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) sc[nt][i] = 0.f;
+                for (int i = 0; i < 4; ++i) sc[nt][i] = 0.f;
 #pragma unroll
-                for (int ks = 0; ks < D / 16; ++ks) {
-                    const int half = ks / 4, ch0 = (ks % 4) * 2;
-#pragma unroll
-                    for (int np = 0; np < NTW / 2; ++np) {  // pairs of 8-row tiles
-                        const int row = warp * kDecRowsPerWarp + np * 16 + (mi >> 1) * 8 + rr;
-                        uint32_t b0, b1, b2, b3;
-                        ldsm_x4(sK + half * C::kHalfBytes + sw128_offset(row, ch0 + (mi & 1)), b0, b1, b2, b3);
-                        mma_bf16_16816(sc[2 * np], qa[ks], b0, b1);
-                        mma_bf16_16816(sc[2 * np + 1], qa[ks], b2, b3);
-                    }
-                }
-                // scale into log2 units, mask, store the group's rows:
-                // c0, c1 -> head gid, c2, c3 -> head gid + 8
-#pragma unroll
-                for (int nt = 0; nt < NTW; ++nt) {
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int hh = gid + (i >> 1) * 8;
-                        const int key = warp * kDecRowsPerWarp + nt * 8 + 2 * tig + (i & 1);
-                        const int spos = pos_of<RING>(j0 + key, it.len, p.R);
-                        const bool vis = spos >= 0 && (!RING || spos > it.len - 1 - p.window);
-                        if (hh < group) sS[hh * kDecRows + key] = vis ? sc[nt][i] * p.scale_log2 : -INFINITY;
-                    }
-                }
+            for (int ks = 0; ks < D / 16; ++ks) {
+                const int half = ks / 4, ch0 = (ks % 4) * 2;
+                const int row = warp * kDecRowsPerWarp + (mi >> 1) * 8 + rr;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(sK + half * C::kHalfBytes + sw128_offset(row, ch0 + (mi & 1)), b0, b1, b2, b3);
+                mma_bf16_16816(sc[0], qa[ks], b0, b1);
+                mma_bf16_16816(sc[1], qa[ks], b2, b3);
             }
-            __syncthreads();
-            // ---- per head (a warp per head): the running max and sum, P = 2^(S - m) in place
-            for (int hh = warp; hh < group; hh += kDecThreads / 32) {
-                float* row = sS + hh * kDecRows;
-                float v[kDecRows / 32];
-                float m = -INFINITY;
+            // ---- online softmax per head: c0, c1 -> head gid, c2, c3 -> head
+            //      gid + 8; the 16 rows of a head sit in one lane quad
+            float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
-                for (int i = 0; i < kDecRows / 32; ++i) {
-                    v[i] = row[lane + 32 * i];
-                    m = fmaxf(m, v[i]);
-                }
-                for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-                const float m_old = sh_m[hh];
-                const float m_new = fmaxf(m_old, m);
-                const float m_use = m_new == -INFINITY ? 0.f : m_new;
-                float l = 0.f;
-#pragma unroll
-                for (int i = 0; i < kDecRows / 32; ++i) {
-                    const float e = ex2_approx(v[i] - m_use);
-                    row[lane + 32 * i] = e;
-                    l += e;
-                }
-                for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-                if (lane == 0) {
-                    const float alpha = m_old == -INFINITY ? 0.f : ex2_approx(m_old - m_use);
-                    sh_alpha[hh] = alpha;
-                    sh_m[hh] = m_new;
-                    sh_l[hh] = sh_l[hh] * alpha + l;
-                }
-            }
-            __syncthreads();
-            // ---- O = O * alpha + P.V over this warp's 16 cache rows (one k-step),
-            //      all D columns; invisible rows carry P = 0 and a zeroed V row
-            {
-                const float a0 = gid < group ? sh_alpha[gid] : 1.f;
-                const float a1 = gid + 8 < group ? sh_alpha[gid + 8] : 1.f;
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                    oc[nt][0] *= a0;
-                    oc[nt][1] *= a0;
-                    oc[nt][2] *= a1;
-                    oc[nt][3] *= a1;
-                }
-            }
-#pragma unroll
-            for (int kk = 0; kk < kDecRowsPerWarp / 16; ++kk) {
-                const int k0 = warp * kDecRowsPerWarp + kk * 16;
-                uint32_t pa[4];  // P rows = heads, columns = cache rows k0..k0+15 (bf16)
+            for (int nt = 0; nt < 2; ++nt) {
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const int hh = gid + (i & 1) * 8;
-                    const int kc = k0 + (i >> 1) * 8 + 2 * tig;
-                    float x0 = 0.f, x1 = 0.f;
-                    if (hh < group) {
-                        x0 = sS[hh * kDecRows + kc];
-                        x1 = sS[hh * kDecRows + kc + 1];
-                    }
-                    pa[i] = pack_bf16x2(x0, x1);
-                }
-#pragma unroll
-                for (int np = 0; np < NT / 2; ++np) {  // pairs of 8-column tiles of V
-                    // matrices: (rows k0..+7, cols n), (rows k0+8..+15, cols n), then n + 8
-                    const int row = k0 + (mi & 1) * 8 + rr;
-                    const int col = np * 16 + (mi >> 1) * 8;  // first head-dim column of the 16-byte chunk
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_trans(sV + (col / 64) * C::kHalfBytes + sw128_offset(row, (col % 64) / 8), b0, b1, b2, b3);
-                    mma_bf16_16816(oc[2 * np], pa, b0, b1);
-                    mma_bf16_16816(oc[2 * np + 1], pa, b2, b3);
+                    const int spos = pos_of<RING>(j0 + nt * 8 + 2 * tig + (i & 1), it.len, p.R);
+                    const bool vis = spos >= 0 && (!RING || spos > it.len - 1 - p.window);
+                    sc[nt][i] = vis ? sc[nt][i] * p.scale_log2 : -INFINITY;
+                    mx[i >> 1] = fmaxf(mx[i >> 1], sc[nt][i]);
                 }
             }
-            fence_proxy_async_smem();  // thread writes to the stage (V zeroing) before its next TMA write
-            __syncthreads();           // the stage and sS are free for the next sub-tile
+            float alpha[2], m_use[2];
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+                mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+                const float m_new = fmaxf(m_run[r], mx[r]);
+                m_use[r] = m_new == -INFINITY ? 0.f : m_new;
+                alpha[r] = ex2_approx(m_run[r] - m_use[r]);  // 0 while nothing was seen
+                m_run[r] = m_new;
+            }
+            float ls[2] = {0.f, 0.f};
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    sc[nt][i] = ex2_approx(sc[nt][i] - m_use[i >> 1]);
+                    ls[i >> 1] += sc[nt][i];
+                }
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                ls[r] += __shfl_xor_sync(0xffffffffu, ls[r], 1);
+                ls[r] += __shfl_xor_sync(0xffffffffu, ls[r], 2);
+                l_run[r] = l_run[r] * alpha[r] + ls[r];
+            }
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                oc[nt][0] *= alpha[0];
+                oc[nt][1] *= alpha[0];
+                oc[nt][2] *= alpha[1];
+                oc[nt][3] *= alpha[1];
+            }
+            // P as the A fragment of rows = heads, k = the warp's 16 cache rows
+            uint32_t pa[4];
+            pa[0] = pack_bf16x2(sc[0][0], sc[0][1]);
+            pa[1] = pack_bf16x2(sc[0][2], sc[0][3]);
+            pa[2] = pack_bf16x2(sc[1][0], sc[1][1]);
+            pa[3] = pack_bf16x2(sc[1][2], sc[1][3]);
+            // ---- O += P.V over the warp's 16 cache rows, all D columns
+#pragma unroll
+            for (int np = 0; np < NT / 2; ++np) {  // pairs of 8-column tiles of V
+                // matrices: (rows k0..+7, cols n), (rows k0+8..+15, cols n), then n + 8
+                const int row = warp * kDecRowsPerWarp + (mi & 1) * 8 + rr;
+                const int col = np * 16 + (mi >> 1) * 8;  // first head-dim column of the 16-byte chunk
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_trans(sV + (col / 64) * C::kHalfBytes + sw128_offset(row, (col % 64) / 8), b0, b1, b2, b3);
+                mma_bf16_16816(oc[2 * np], pa, b0, b1);
+                mma_bf16_16816(oc[2 * np + 1], pa, b2, b3);
+            }
+            // the warp is done with the stage (its V-row writes ordered before
+            // the stage's next TMA write)
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bar_empty[st]));
         }
-        if (!ok) break;
-        // ---- sum the four warps' partial O through shared memory: [warp][head][D]
-        //      in the K tile of the stage consumed last
-        float* sO = reinterpret_cast<float*>(smem + ((consumed - 1) % kDecStages) * C::kStageBytes);
+        // every thread of the CTA reaches this barrier, and all stop together if
+        // any wait gave up
+        if (!__syncthreads_and(ok)) break;
+        // ---- the four warps' partials: [warp][head][D + 2] in shared memory
+        {
+            float* mw = sM + warp * group * (D + 2);
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
+            for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int hh = gid + (i >> 1) * 8;
-                const int d = nt * 8 + 2 * tig + (i & 1);
-                if (hh < group) sO[(warp * group + hh) * D + d] = oc[nt][i];
+                for (int i = 0; i < 4; ++i) {
+                    const int hh = gid + (i >> 1) * 8;
+                    const int d = nt * 8 + 2 * tig + (i & 1);
+                    if (hh < group) mw[hh * (D + 2) + d] = oc[nt][i];
+                }
             }
+            if (tig == 0) {
+#pragma unroll
+                for (int r = 0; r < 2; ++r) {
+                    const int hh = gid + 8 * r;
+                    if (hh < group) {
+                        mw[hh * (D + 2) + D] = m_run[r];
+                        mw[hh * (D + 2) + D + 1] = l_run[r];
+                    }
+                }
+            }
+        }
+        __syncthreads();
+        if (tid < group) {  // per head: M = max_w m_w, L = sum_w 2^(m_w - M) l_w
+            float M = -INFINITY;
+#pragma unroll
+            for (int wv = 0; wv < 4; ++wv) M = fmaxf(M, sM[(wv * group + tid) * (D + 2) + D]);
+            float L = 0.f;
+#pragma unroll
+            for (int wv = 0; wv < 4; ++wv) {
+                const float mv = sM[(wv * group + tid) * (D + 2) + D];
+                const float wgt = (M == -INFINITY || mv == -INFINITY) ? 0.f : ex2_approx(mv - M);
+                sh_wm[wv][tid] = wgt;
+                L += wgt * sM[(wv * group + tid) * (D + 2) + D + 1];
+            }
+            sh_M[tid] = M;
+            sh_L[tid] = L;
         }
         __syncthreads();
         if (it.nused == 1) {  // the whole cache in this item: normalise and write the output
@@ -344,12 +368,12 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
                 const int hh = i / D, d = i % D;
                 float acc = 0.f;
 #pragma unroll
-                for (int wv = 0; wv < kDecThreads / 32; ++wv) acc += sO[(wv * group + hh) * D + d];
-                const float L = sh_l[hh];
+                for (int wv = 0; wv < 4; ++wv) acc += sh_wm[wv][hh] * sM[(wv * group + hh) * (D + 2) + d];
+                const float L = sh_L[hh];
                 const __nv_bfloat16 bv = __float2bfloat16_rn(L > 0.f ? acc / L : 0.f);
                 p.out[(static_cast<int64_t>(it.r) * p.Hq + h0 + hh) * D + d] = *reinterpret_cast<const logo_bf16*>(&bv);
             }
-            __syncthreads();  // sO and sh_m / sh_l are reused by the next item
+            __syncthreads();  // the merge buffer is reused by the next item
             continue;
         }
         // ---- a chunk of a longer cache: partial result, then the last chunk merges
@@ -357,12 +381,12 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
             const int hh = i / D, d = i % D;
             float acc = 0.f;
 #pragma unroll
-            for (int wv = 0; wv < kDecThreads / 32; ++wv) acc += sO[(wv * group + hh) * D + d];
+            for (int wv = 0; wv < 4; ++wv) acc += sh_wm[wv][hh] * sM[(wv * group + hh) * (D + 2) + d];
             float* dst = p.part + ((static_cast<int64_t>(it.r) * p.Hq + h0 + hh) * p.nchunk + it.c) * (D + 2);
             dst[d] = acc;
             if (d == 0) {
-                dst[D] = sh_m[hh];
-                dst[D + 1] = sh_l[hh];
+                dst[D] = sh_M[hh];
+                dst[D + 1] = sh_L[hh];
             }
         }
         __syncthreads();  // every partial of this chunk is written
@@ -375,7 +399,7 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
         __syncthreads();
         if (sh_last) {
             // M = max_c m_c, L = sum_c 2^(m_c - M) l_c, o = sum_c 2^(m_c - M) o_c / L,
-            // per head: the weights first (into sS), then thread (head, d) adds the chunks
+            // per head: the weights first (into sW), then thread (head, d) adds the chunks
             for (int i = tid; i < group * it.nused; i += kDecThreads) {
                 const int hh = i / it.nused;
                 const float* base = p.part + (static_cast<int64_t>(it.r) * p.Hq + h0 + hh) * p.nchunk * (D + 2);
@@ -383,13 +407,13 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
                 for (int c = 0; c < it.nused; ++c) M = fmaxf(M, __ldcg(base + c * (D + 2) + D));
                 const int c = i % it.nused;
                 const float m = __ldcg(base + c * (D + 2) + D);
-                sS[hh * it.nused + c] = m == -INFINITY ? 0.f : ex2_approx(m - M);
+                sW[hh * it.nused + c] = m == -INFINITY ? 0.f : ex2_approx(m - M);
             }
             __syncthreads();
             for (int i = tid; i < group * D; i += kDecThreads) {
                 const int hh = i / D, d = i % D;
                 const float* base = p.part + (static_cast<int64_t>(it.r) * p.Hq + h0 + hh) * p.nchunk * (D + 2);
-                const float* wts = sS + hh * it.nused;
+                const float* wts = sW + hh * it.nused;
                 float o = 0.f, L = 0.f;
                 for (int c = 0; c < it.nused; ++c) {
                     const float wc = wts[c];
@@ -400,7 +424,7 @@ __global__ void __launch_bounds__(kDecThreads, 2) decode_attn_kernel(const __gri
                 p.out[(static_cast<int64_t>(it.r) * p.Hq + h0 + hh) * D + d] = *reinterpret_cast<const logo_bf16*>(&bv);
             }
         }
-        __syncthreads();  // sO, sS and sh_m / sh_l are reused by the next item
+        __syncthreads();  // sW and the merge buffer are reused by the next item
     }
     if (!ok && tid == 0) {  // let copies already issued land before the CTA exits
         for (int k = consumed; k < issued; ++k) mbar_wait_drain(smem_u32(&bar_full[k % kDecStages]), (k / kDecStages) & 1);
@@ -449,21 +473,29 @@ int launch_decode(DecParams& prm, cudaStream_t st)
 {
     static bool attr_done = false;  // benign race: setting the attribute twice is harmless
     if (!attr_done) {
-        if (set_smem_limit(decode_attn_kernel<D, RING>, DecCfg<D>::kSmemBytes) != cudaSuccess) return LOGO_ERR_CUDA;
+        if (set_smem_limit(decode_attn_kernel<D, RING>, DecCfg<D>::smem_bytes(kDecMaxGroup)) != cudaSuccess)
+            return LOGO_ERR_CUDA;
         attr_done = true;
     }
-    // as many resident CTAs as fit (each keeps two sub-tiles' K/V loads in flight)
-    static int per_sm = 0;
-    if (per_sm == 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_attn_kernel<D, RING>, kDecThreads,
-                                                                      DecCfg<D>::kSmemBytes) != cudaSuccess ||
-                        per_sm < 1))
-        per_sm = 2;
+    // as many resident CTAs as fit (each keeps up to three sub-tiles' K/V loads in
+    // flight); the merge buffer, and so the fit, depends on the group size
+    const int group = prm.Hq / prm.Hkv;
+    const int smem = DecCfg<D>::smem_bytes(group);
+    static int per_sm_of[kDecMaxGroup + 1] = {};
+    int per_sm = per_sm_of[group];
+    if (per_sm == 0) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_attn_kernel<D, RING>, kDecThreads, smem) !=
+                cudaSuccess ||
+            per_sm < 1)
+            per_sm = 1;
+        per_sm_of[group] = per_sm;
+    }
     const long long items = static_cast<long long>(prm.B) * prm.Hkv * prm.nchunk;
     const int grid = static_cast<int>(std::max(1ll, std::min(items, static_cast<long long>(per_sm) * device_sm_count())));
     if (prm.nchunk > 1 &&  // the chunk counters start at zero
         cudaMemsetAsync(prm.done, 0, static_cast<size_t>(prm.B) * prm.Hkv * sizeof(int32_t), st) != cudaSuccess)
         return LOGO_ERR_CUDA;
-    decode_attn_kernel<D, RING><<<grid, kDecThreads, DecCfg<D>::kSmemBytes, st>>>(prm);
+    decode_attn_kernel<D, RING><<<grid, kDecThreads, smem, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 
