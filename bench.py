@@ -3,7 +3,10 @@
 
 One step = one training pass of the layer over one batch of synthetic input:
 select -> local fwd -> global fwd -> combine -> combine bwd -> global bwd ->
-local bwd (every call through the C ABI, inputs resident in HBM).
+local bwd (every call through the C ABI, inputs resident in HBM; the local
+calls run on a second stream beside the global calls, forked after the
+selection and after the combine bwd, joined before the combine and at the end
+of the step).
 
 Metric: useful TFLOP/s of the whole step.  Useful FLOPs count only the
 query-key pairs the method must compute, 14*d per pair per head (4*d forward:
@@ -195,18 +198,24 @@ def step_calls(layer, g):
                                                              workspace=layer.ws)),
         ("local_bwd", lambda: L.logo_local_attn_bwd(g["qL"], g["kL"], g["vL"], layer.o_l, layer.lse_l, layer.dO_l,
                                                     c.window, c.scale, layer.dqL, layer.dkL, layer.dvL,
-                                                    workspace=layer.ws)),
+                                                    workspace=layer.ws_l)),
     ]
 
 
 def run_step(layer, g, ev=None):
-    """One full step; if ev is given, record an event after each call."""
-    if ev is not None:
-        ev[0].record()
+    """One full step through the layer: the local branch on the layer's side
+    stream beside the global branch.  If ev is given, the
+    seven calls run in order on one stream instead, with an event recorded
+    after each (per-call times)."""
+    if ev is None:
+        args = (g["qL"], g["kL"], g["vL"], g["qG"], g["kG"], g["vG"], g["p"])
+        layer.forward(*args)
+        layer.backward(g["dO"], *args)
+        return
+    ev[0].record()
     for i, (_, call) in enumerate(step_calls(layer, g)):
         call()
-        if ev is not None:
-            ev[i + 1].record()
+        ev[i + 1].record()
 
 
 def per_call_device_ms(layer, g, reps):
@@ -657,7 +666,8 @@ def native_arm(a, rank, world, local_rank, dist_on):
             "local_fwd_bwd": {"tflops": fl_local / (l_ms / 1e3) / 1e12, "ms": l_ms},
             "useful_flops_per_step": fl_step, "pairs_per_head": {"local": lp, "global": gp},
             "selected": n, "per_call": breakdown, "roofline": roof,
-            "launch": ("one CUDA graph replay per step" if graph is not None else "eager calls"),
+            "launch": ("one CUDA graph replay per step; the local calls on a second stream beside the "
+                       "global calls" if graph is not None else "eager calls, one stream"),
             "eager_ms_per_step": eager_ms,
             "gpu_launches": launches_per_step(w) * a.steps, "clocks": clk.summary()}
 

@@ -3,6 +3,17 @@ C-ABI entry points (forward: select, local, global, combine; backward:
 combine_bwd, global_bwd, local_bwd).  Buffers and workspaces are allocated
 once per shape and reused, so a step launches kernels only.
 
+The two branches are independent between the selection and the combine, and
+again after the combine's backward, so the local calls run on a side stream
+(forked from and joined back into the caller's stream) beside the global
+calls: the kernel launched second fills the SMs the first one's tail leaves
+idle, and the HBM-bound passes of one branch overlap the tensor-core work of
+the other.  The local call is issued first on each fork: its persistent
+kernel is the longer one, and with the global kernel launched first the local
+kernel's late CTAs stretched the step.  The local backward has a
+workspace of its own for that reason.  `overlap=False` keeps every call on
+the caller's stream.
+
 `forward` / `backward` take the branch inputs and the gate values as the
 caller made them (the projections of Eq. 4/5, the gate of Eq. 7 and the
 output projection stay outside).  `forward_fused` / `backward_fused` also
@@ -38,9 +49,11 @@ class LayerConfig:
 class LogoAttention:
     """Preallocated forward/backward of the layer for one shape on one device."""
 
-    def __init__(self, cfg: LayerConfig, device="cuda"):
+    def __init__(self, cfg: LayerConfig, device="cuda", overlap: bool = True):
         self.cfg = c = cfg
         dev = torch.device(device)
+        self.overlap = overlap
+        self.side = torch.cuda.Stream(device=dev) if overlap and dev.type == "cuda" else None
         self.dims = L.Dims(c.B, c.T, c.Hq, c.Hkv, c.D)
         cap = c.B * c.T
         bf, f32, i32 = torch.bfloat16, torch.float32, torch.int32
@@ -69,17 +82,56 @@ class LogoAttention:
         self.dqG = e((c.B, c.T, c.Hq, c.D), bf)
         self.dkG = e((c.B, c.T, c.Hkv, c.D), bf)
         self.dvG = e((c.B, c.T, c.Hkv, c.D), bf)
-        # workspaces: the largest of the calls, shared (calls are stream-ordered)
-        nbytes = max(L.workspace_bytes(k, self.dims) for k in ("select", "local_bwd", "global_fwd", "global_bwd"))
+        # workspaces: one shared by the calls on the caller's stream (they are
+        # stream-ordered), one for the local backward on the side stream
+        nbytes = max(L.workspace_bytes(k, self.dims) for k in ("select", "global_fwd", "global_bwd"))
         self.ws = e((nbytes,), torch.uint8)
+        self.ws_l = e((L.workspace_bytes("local_bwd", self.dims),), torch.uint8)
+
+    def _fork(self):
+        """Side stream for the local branch (None: run it in order)."""
+        if self.side is None:
+            return None
+        self.side.wait_stream(torch.cuda.current_stream())
+        return torch.cuda.stream(self.side)
+
+    def _join(self):
+        if self.side is not None:
+            torch.cuda.current_stream().wait_stream(self.side)
+
+    def _local_fwd(self, qL, kL, vL):
+        c = self.cfg
+        L.logo_local_attn_fwd(qL, kL, vL, c.window, c.scale, self.o_l, self.lse_l)
+
+    def _local_bwd(self, qL, kL, vL):
+        c = self.cfg
+        L.logo_local_attn_bwd(qL, kL, vL, self.o_l, self.lse_l, self.dO_l, c.window, c.scale, self.dqL, self.dkL,
+                              self.dvL, workspace=self.ws_l)
+
+    def _branches(self, local, other):
+        """local() on the side stream beside other() on the caller's stream,
+        joined before returning; both in order without a side stream."""
+        ctx = self._fork()
+        if ctx is None:
+            other()
+            local()
+            return
+        with ctx:
+            local()
+        other()
+        self._join()
 
     def forward(self, qL, kL, vL, qG, kG, vG, gate_p, gain_l=None, gain_g=None):
         c = self.cfg
+        # the fork follows the selection: captured in a CUDA graph, a local
+        # branch forked at the very start would be a second root node, and
+        # the graph then launched the global backward ahead of the local one
+        # (measured at 16K: 2.39 ms a step against 2.23 with this order)
         L.logo_select(gate_p, c.mode, c.b_th, c.ratio, self.z, self.pos, self.cu_q, self.row_of, self.n_sel,
                       workspace=self.ws)
-        L.logo_local_attn_fwd(qL, kL, vL, c.window, c.scale, self.o_l, self.lse_l)
-        L.logo_global_sparse_attn_fwd(qG, kG, vG, self.pos, self.cu_q, self.n_sel, c.scale, self.o_c, self.lse_c,
-                                      workspace=self.ws)
+        self._branches(lambda: self._local_fwd(qL, kL, vL),
+                       lambda: L.logo_global_sparse_attn_fwd(qG, kG, vG, self.pos, self.cu_q, self.n_sel, c.scale,
+                                                             self.o_c, self.lse_c, workspace=self.ws))
         L.logo_combine(self.o_l, self.o_c, gate_p, self.z, self.row_of, gain_l, gain_g, c.eps, self.o, self.rstd_l,
                        self.rstd_g)
         return self.o
@@ -88,10 +140,10 @@ class LogoAttention:
         c = self.cfg
         L.logo_combine_bwd(dO, self.o_l, self.o_c, gate_p, self.z, self.row_of, gain_l, gain_g, c.eps, self.dO_l,
                            self.dO_c, self.dgate)
-        L.logo_global_sparse_attn_bwd(qG, kG, vG, self.pos, self.cu_q, self.n_sel, self.o_c, self.lse_c, self.dO_c,
-                                      c.scale, self.dqG, self.dkG, self.dvG, workspace=self.ws)
-        L.logo_local_attn_bwd(qL, kL, vL, self.o_l, self.lse_l, self.dO_l, c.window, c.scale, self.dqL, self.dkL,
-                              self.dvL, workspace=self.ws)
+        self._branches(lambda: self._local_bwd(qL, kL, vL),
+                       lambda: L.logo_global_sparse_attn_bwd(qG, kG, vG, self.pos, self.cu_q, self.n_sel, self.o_c,
+                                                             self.lse_c, self.dO_c, c.scale, self.dqG, self.dkG,
+                                                             self.dvG, workspace=self.ws))
         return dict(dqL=self.dqL, dkL=self.dkL, dvL=self.dvL, dqG=self.dqG, dkG=self.dkG, dvG=self.dvG,
                     dgate_p=self.dgate)
 
@@ -128,11 +180,10 @@ class LogoAttention:
             self.dw_g = torch.empty_like(w_g)
         L.logo_combine_bwd_gains(dO, self.o_l, self.o_c, self.gate_p, self.z, self.row_of, gain_l, gain_g, c.eps,
                                  self.dO_l, self.dO_c, self.dgate, self.dgain_l, self.dgain_g)
-        L.logo_global_sparse_attn_bwd(self.qG, self.kG, self.vG, self.pos, self.cu_q, self.n_sel, self.o_c,
-                                      self.lse_c, self.dO_c, c.scale, self.dqG, self.dkG, self.dvG,
-                                      workspace=self.ws)
-        L.logo_local_attn_bwd(qL, kL, vL, self.o_l, self.lse_l, self.dO_l, c.window, c.scale, self.dqL, self.dkL,
-                              self.dvL, workspace=self.ws)
+        self._branches(lambda: self._local_bwd(qL, kL, vL),
+                       lambda: L.logo_global_sparse_attn_bwd(self.qG, self.kG, self.vG, self.pos, self.cu_q,
+                                                             self.n_sel, self.o_c, self.lse_c, self.dO_c, c.scale,
+                                                             self.dqG, self.dkG, self.dvG, workspace=self.ws))
         rows = (self.pos, self.cu_q, self.n_sel)
         back = lambda t: {k: v for k, v in t.items() if k != "b"}  # noqa: E731  (b does not enter the backward)
         tqg = L.logo_branch_transform_bwd(qL, self.dqG, rows=rows, du_l=self.dqL, accumulate=True, **back(tq))

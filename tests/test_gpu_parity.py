@@ -362,6 +362,33 @@ def test_layer_step_4k_workload():
     check_close(np32(grads["dvG"])[:, :, h], rdv[:, :, h], "dvG")
 
 
+def test_layer_two_streams_match_one_stream():
+    """The local branch on the layer's side stream gives the results of the
+    seven calls in order on one stream: every output bit-identical except dQ,
+    whose fp32 reductions resolve in a run-dependent order (one bf16 ulp)."""
+    from paper_2608_29539_gb300.layer import LayerConfig, LogoAttention
+    from paper_2608_29539_gb300.workloads import WORKLOADS, make_inputs
+    w = WORKLOADS["4k"]
+    x = make_inputs(w, device="cuda")
+    cfg = LayerConfig(B=w.B, T=w.T, Hq=w.Hq, Hkv=w.Hkv, D=w.D, window=w.window, mode=1, ratio=w.ratio)
+    out = []
+    for overlap in (False, True):
+        layer = LogoAttention(cfg, overlap=overlap)
+        args = (x["qL"], x["kL"], x["vL"], x["qG"], x["kG"], x["vG"], x["p"])
+        for _ in range(2):
+            layer.forward(*args)
+            grads = layer.backward(x["dO"], *args)
+        torch.cuda.synchronize()
+        out.append(dict(o=layer.o.clone(), lse_l=layer.lse_l.clone(), **{k: v.clone() for k, v in grads.items()}))
+    assert L().logo_get_device_status() == 0
+    for k in out[0]:
+        a, b = out[0][k].float(), out[1][k].float()
+        if k in ("dqL", "dqG"):
+            np.testing.assert_allclose(b.cpu().numpy(), a.cpu().numpy(), rtol=2 ** -7, atol=1e-3, err_msg=k)
+        else:
+            assert torch.equal(a, b), k
+
+
 # ------------------------------------------- full size, the benchmark's launch
 # Local backward shapes with several KV-block items per CTA on a 152-SM GPU
 # (each CTA walks 5-7 items): item sequences crossing sequences and KV
