@@ -845,10 +845,16 @@ __global__ void __launch_bounds__(Bwd2Cfg::kThreads, 1) attn_bwd2_kernel(const _
             const int key = it.j * kBN + t;
             const int64_t kv_off = ((static_cast<int64_t>(it.b) * p.T + key) * p.Hkv + it.kvh) * D;
             if (it.ntiles == 0) {
-                if (key < p.T) {
-                    for (int c = 0; c < D; c += 8) {
-                        *reinterpret_cast<uint4*>(p.dk + kv_off + c) = make_uint4(0, 0, 0, 0);
-                        *reinterpret_cast<uint4*>(p.dv + kv_off + c) = make_uint4(0, 0, 0, 0);
+                // no selected query sees the block: zero dK, dV rows, two whole
+                // rows (16 lanes x 16 bytes each) per warp store, this warp's 32 keys
+                static_assert(D == 128, "two rows of 16 vectors per warp store");
+                for (int r = quad * 32 + (lane >> 4); r < quad * 32 + 32; r += 2) {
+                    const int kr = it.j * kBN + r;
+                    if (kr < p.T) {
+                        const int64_t off =
+                            ((static_cast<int64_t>(it.b) * p.T + kr) * p.Hkv + it.kvh) * D + (lane & 15) * 8;
+                        *reinterpret_cast<uint4*>(p.dk + off) = make_uint4(0, 0, 0, 0);
+                        *reinterpret_cast<uint4*>(p.dv + off) = make_uint4(0, 0, 0, 0);
                     }
                 }
                 continue;
