@@ -48,8 +48,8 @@ L2_BYTES = 129 * 1024 * 1024
 # source is unchanged (see profiles/).
 TRAFFIC = {
     # attn_bwd2_kernel, 16K workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, one launch each)
-    ("local_bwd", "719cf024947d3e17"): 824331776 + 479615232,
-    ("global_bwd", "719cf024947d3e17"): 470104320 + 431910400,
+    ("local_bwd", "f716c69b384b4931"): 824986112 + 482090752,
+    ("global_bwd", "f716c69b384b4931"): 476076288 + 432424704,
 }
 
 
