@@ -218,33 +218,37 @@ def run_step(layer, g, ev=None):
         ev[i + 1].record()
 
 
-def per_call_device_ms(layer, g, reps):
-    """Device time of each call: the call captured `reps` times back to back as
-    one CUDA graph, one replay timed with CUDA events on the launching stream,
-    divided by `reps`.  (Timing single eager calls would add the host's launch
-    time of a small call to its duration.)  Every call is idempotent on the
-    step's buffers, so repeating it leaves the state of the step unchanged."""
-    out = {}
-    for name, call in step_calls(layer, g):
-        side = torch.cuda.Stream()
-        side.wait_stream(torch.cuda.current_stream())
-        with torch.cuda.stream(side):
+def graph_ms(call, reps=20):
+    """Device time of call(): one eager call on a side stream, then the call
+    captured `reps` times back to back as one CUDA graph, one warm-up replay and
+    one replay timed with CUDA events on the launching stream, divided by
+    `reps`.  (Timing eager calls would add the host's launch time of a small
+    call to its duration.)"""
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        call()
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for _ in range(reps):
             call()
-        torch.cuda.current_stream().wait_stream(side)
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            for _ in range(reps):
-                call()
-        graph.replay()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        torch.cuda.synchronize()
-        e0.record()
-        graph.replay()
-        e1.record()
-        torch.cuda.synchronize()
-        out[name] = e0.elapsed_time(e1) / reps
-        del graph
-    return out
+    graph.replay()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    del graph
+    return e0.elapsed_time(e1) / reps
+
+
+def per_call_device_ms(layer, g, reps):
+    """Device time of each call of the step (graph_ms).  Every call is
+    idempotent on the step's buffers, so repeating it leaves the state of the
+    step unchanged."""
+    return {name: graph_ms(call, reps) for name, call in step_calls(layer, g)}
 
 
 def layer_for(w, device):
@@ -393,17 +397,10 @@ def routing_bench(layer, x, w, dev):
         L.logo_select_device_threshold(x["p"], b_dev, *rl_bufs, workspace=layer.ws)
         L.logo_budget_update(rl_bufs[4], w.B, w.T, w.ratio, 2.0 ** -11, b_dev, f_out=f_dev)
 
-    for _ in range(3):
-        routing_step()
-    torch.cuda.synchronize()
-    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    r0.record()
-    for _ in range(50):
-        routing_step()
-    r1.record()
-    torch.cuda.synchronize()
-    return {"us_per_step": r0.elapsed_time(r1) / 50 * 1e3, "launches_per_step": 4,
-            "note": "logo_select_device_threshold + logo_budget_update, no host sync"}
+    # each step reads the threshold the previous one wrote: 50 steps in one graph
+    return {"us_per_step": graph_ms(routing_step, 50) * 1e3, "launches_per_step": 4,
+            "note": "logo_select_device_threshold + logo_budget_update, no host sync; device time per step "
+                    "(50 steps captured as one CUDA graph)"}
 
 
 def fusions_bench(layer, x, w, dev, pk):
@@ -430,17 +427,7 @@ def fusions_bench(layer, x, w, dev, pk):
     dgg = torch.empty_like(dgl)
     n = int(layer.n_sel[0])
 
-    def timed(fn, reps=20):
-        for _ in range(3):
-            fn()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for _ in range(reps):
-            fn()
-        e1.record()
-        torch.cuda.synchronize()
-        return e0.elapsed_time(e1) / reps
+    timed = graph_ms  # device time per call
 
     gate = lambda: L.logo_gate_select(xin, wg, c.mode, c.b_th, c.ratio, *bufs, workspace=layer.ws)  # noqa: E731
     gate_bwd = lambda: L.logo_gate_bwd(xin, wg, bufs[0], layer.dgate, dx=dxin, accumulate=True, dw_g=dw,  # noqa: E731
@@ -534,17 +521,8 @@ def decode_bench(dev, pk):
         main.wait_stream(aux)
         L.logo_combine(o_l.view(B, 1, Hq, D), o_c, p, zz, ro, None, None, 1e-6, o, rl, rg)
 
-    def timed(sel, reps=20):
-        for _ in range(3):
-            step(sel)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for _ in range(reps):
-            step(sel)
-        e1.record()
-        torch.cuda.synchronize()
-        return e0.elapsed_time(e1) / reps
+    def timed(sel, reps=20):  # device time per step, both streams inside one graph
+        return graph_ms(lambda: step(sel), reps)
 
     sparse_ms = timed(sparse_sel)
     dense_ms = timed(dense_sel)

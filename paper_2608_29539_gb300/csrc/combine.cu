@@ -8,9 +8,9 @@
 // loads before any arithmetic (so each thread keeps VPT to 3*VPT loads in
 // flight), and the D/8 lanes of a head reduce their sums with warp shuffles.
 // The backward sums dp_t over every head of the token in shared memory, and
-// the gain gradients over tokens in registers (fixed vectors per thread), then
-// per block into a workspace that a second kernel sums in a fixed order
-// (colsum.cuh: deterministic).  All arithmetic is fp32; inputs and outputs bf16.
+// the gain gradients over the block's tokens in shared-memory slots that only
+// the thread owning the vector touches, then per block into a workspace that a
+// second kernel sums in a fixed order (colsum.cuh: deterministic).  All arithmetic is fp32; inputs and outputs bf16.
 // The kernels are bound as much by instruction issue as by HBM: without gains
 // (both NULL, i.e. 1) a separate instantiation drops the gain loads and the
 // unit multiplies and does the elementwise work as f32x2 pairs.
@@ -111,6 +111,23 @@ __device__ __forceinline__ Vec8 axpby8(const Vec8& x, float a, const Vec8* y, fl
     return r;
 }
 
+// Gain-gradient accumulators of the backward, in shared memory: float4 slot
+// (branch * 2 + half) * nvec + v holds elements 4 half .. 4 half + 3 of vector
+// v's sums.  Only the thread that owns vector v touches its slots, and a
+// warp's 32 consecutive vectors are 32 consecutive float4 (no bank conflicts).
+// In registers they took 32 more per thread (at Hq*D = 4096), which cut the
+// resident blocks per SM, and with them the loads in flight, by half.
+__device__ __forceinline__ void acc_add8(float4* sh, int nvec, int branch, int v, const Vec8& c)
+{
+    float4* p0 = sh + (branch * 2) * nvec + v;
+    float4* p1 = p0 + nvec;
+    float4 a = *p0, b = *p1;
+    a.x += c.v[0]; a.y += c.v[1]; a.z += c.v[2]; a.w += c.v[3];
+    b.x += c.v[4]; b.y += c.v[5]; b.z += c.v[6]; b.w += c.v[7];
+    *p0 = a;
+    *p1 = b;
+}
+
 // Sum over the `width` consecutive lanes (a power of two <= 32) of one head.
 __device__ __forceinline__ float head_sum(float x, int width)
 {
@@ -189,9 +206,10 @@ __global__ void __launch_bounds__(kThreads) combine_fwd_kernel(
 }
 
 // part (DGAIN): [gridDim.x][2][H*D] float32 per-block sums of the local and
-// global gain gradients.
+// global gain gradients, accumulated in dynamic shared memory (4 * nvec float4,
+// see acc_add8) over the block's tokens in increasing order.
 template <int VPT, bool DGAIN, bool UNIT>
-__global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
+__global__ void __launch_bounds__(kThreads, DGAIN && VPT <= 2 ? 3 : 1) combine_bwd_kernel(
     const logo_bf16* __restrict__ dO, const logo_bf16* __restrict__ o_l, const logo_bf16* __restrict__ o_c,
     const float* __restrict__ gate_p, const uint8_t* __restrict__ z, const int32_t* __restrict__ row_of,
     const float* __restrict__ gain_l, const float* __restrict__ gain_g, float eps, logo_bf16* __restrict__ dO_l,
@@ -201,12 +219,15 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
     const int vpr = D / 8;
     const int nvec = H * vpr;
     const float inv_d = 1.0f / static_cast<float>(D);
-    float accL[DGAIN ? VPT : 1][8], accG[DGAIN ? VPT : 1][8];
+    extern __shared__ float4 sh_acc[];
     if (DGAIN) {
 #pragma unroll
-        for (int k = 0; k < VPT; ++k)
+        for (int k = 0; k < VPT; ++k) {
+            const int v = threadIdx.x + k * kThreads;
+            if (v < nvec)
 #pragma unroll
-            for (int i = 0; i < 8; ++i) accL[k][i] = accG[k][i] = 0.f;
+                for (int s = 0; s < 4; ++s) sh_acc[s * nvec + v] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
     }
     int n_sel_seen = 0;
     for (int64_t bt = blockIdx.x; bt < ntok; bt += gridDim.x) {
@@ -240,8 +261,10 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
                 const float cl = r_l * r_l * r_l * xgdy * inv_d;
                 if (active) store_bf16x8(dO_l + (bt * nvec + v) * 8, axpby8(g, r_l * wl, &xl, -cl));
                 if constexpr (DGAIN) {  // d gain_l = dy * x r
+                    Vec8 c;
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) accL[k][i] += g.v[i] * wl * xl.v[i] * r_l;
+                    for (int i = 0; i < 8; ++i) c.v[i] = g.v[i] * wl * xl.v[i] * r_l;
+                    if (active) acc_add8(sh_acc, nvec, 0, v, c);
                 }
                 if (sel) {
                     const Vec8 xg = unpack8(rg[k]);
@@ -251,8 +274,10 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
                     const float cg = r_g * r_g * r_g * xgdyg * inv_d;
                     if (active) store_bf16x8(dO_c + (row * nvec + v) * 8, axpby8(g, r_g * pt, &xg, -cg));
                     if constexpr (DGAIN) {
+                        Vec8 c;
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) accG[k][i] += g.v[i] * pt * xg.v[i] * r_g;
+                        for (int i = 0; i < 8; ++i) c.v[i] = g.v[i] * pt * xg.v[i] * r_g;
+                        if (active) acc_add8(sh_acc, nvec, 1, v, c);
                     }
                     // dp += dO . (xg r_g - xl r_l)
                     const uint64_t rg2 = f2_pack(r_g, r_g), rl2 = f2_pack(-r_l, -r_l);
@@ -281,9 +306,11 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
 #pragma unroll
             for (int i = 0; i < 8; ++i) dxl.v[i] = r_l * gl.v[i] * g.v[i] * wl - xl.v[i] * cl;
             if (active) store_bf16x8(dO_l + (bt * nvec + v) * 8, dxl);
-            if (DGAIN) {  // d gain_l = dy * x r
+            if constexpr (DGAIN) {  // d gain_l = dy * x r
+                Vec8 c;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) accL[k][i] += g.v[i] * wl * xl.v[i] * r_l;
+                for (int i = 0; i < 8; ++i) c.v[i] = g.v[i] * wl * xl.v[i] * r_l;
+                if (active) acc_add8(sh_acc, nvec, 0, v, c);
             }
             if (sel) {
                 const Vec8 xg = unpack8(rg[k]);
@@ -305,9 +332,11 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
                     dp_acc += g.v[i] * (xg.v[i] * r_g * gg.v[i] - xl.v[i] * r_l * gl.v[i]);
                 }
                 if (active) store_bf16x8(dO_c + (row * nvec + v) * 8, dxg);
-                if (DGAIN) {
+                if constexpr (DGAIN) {
+                    Vec8 c;
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) accG[k][i] += g.v[i] * pt * xg.v[i] * r_g;
+                    for (int i = 0; i < 8; ++i) c.v[i] = g.v[i] * pt * xg.v[i] * r_g;
+                    if (active) acc_add8(sh_acc, nvec, 1, v, c);
                 }
             }
         }
@@ -341,9 +370,10 @@ __global__ void __launch_bounds__(kThreads) combine_bwd_kernel(
             const int v = threadIdx.x + k * kThreads;
             if (v < nvec) {
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    pl[v * 8 + i] = accL[k][i];
-                    pl[hd + v * 8 + i] = accG[k][i];
+                for (int br = 0; br < 2; ++br) {
+                    float4* dst = reinterpret_cast<float4*>(pl + br * hd + v * 8);
+                    dst[0] = sh_acc[(br * 2) * nvec + v];
+                    dst[1] = sh_acc[(br * 2 + 1) * nvec + v];
                 }
             }
         }
@@ -360,13 +390,25 @@ int vec_per_thread(const logo_dims& d)
 // One wave of resident blocks (the grid-stride loop gives every block the
 // same number of tokens), capped by the token count.
 template <typename K>
-int64_t wave_blocks(K kernel, int64_t ntok)
+int64_t wave_blocks(K kernel, int64_t ntok, size_t smem = 0)
 {
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, 0) != cudaSuccess || per_sm < 1)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem) != cudaSuccess || per_sm < 1)
         per_sm = 1;
     const int64_t cap = static_cast<int64_t>(device_sm_count()) * per_sm;
     return ntok < cap ? ntok : cap;
+}
+
+// Dynamic shared memory of the gain-gradient backward: its accumulators.
+size_t gains_smem(const logo_dims& d) { return static_cast<size_t>(4) * (d.Hq * d.D / 8) * sizeof(float4); }
+
+// The gain variant may need more than the default 48 KB of dynamic shared
+// memory (64 KB at Hq*D = 8192); the attribute is set before any occupancy
+// query or launch of it.
+template <typename K>
+bool gains_smem_ok(K kernel)
+{
+    return set_smem_limit(kernel, 4 * kMaxVecGains * static_cast<int>(sizeof(float4))) == cudaSuccess;
 }
 
 // Blocks of the gain-gradient backward (one partial row each): the larger of
@@ -374,16 +416,23 @@ int64_t wave_blocks(K kernel, int64_t ntok)
 int64_t gains_blocks(const logo_dims& d)
 {
     const int64_t ntok = static_cast<int64_t>(d.B) * d.T;
+    const size_t smem = gains_smem(d);
     switch (vec_per_thread(d)) {
         case 1:
-            return std::max(wave_blocks(combine_bwd_kernel<1, true, false>, ntok),
-                            wave_blocks(combine_bwd_kernel<1, true, true>, ntok));
+            gains_smem_ok(combine_bwd_kernel<1, true, false>);
+            gains_smem_ok(combine_bwd_kernel<1, true, true>);
+            return std::max(wave_blocks(combine_bwd_kernel<1, true, false>, ntok, smem),
+                            wave_blocks(combine_bwd_kernel<1, true, true>, ntok, smem));
         case 2:
-            return std::max(wave_blocks(combine_bwd_kernel<2, true, false>, ntok),
-                            wave_blocks(combine_bwd_kernel<2, true, true>, ntok));
+            gains_smem_ok(combine_bwd_kernel<2, true, false>);
+            gains_smem_ok(combine_bwd_kernel<2, true, true>);
+            return std::max(wave_blocks(combine_bwd_kernel<2, true, false>, ntok, smem),
+                            wave_blocks(combine_bwd_kernel<2, true, true>, ntok, smem));
         default:
-            return std::max(wave_blocks(combine_bwd_kernel<4, true, false>, ntok),
-                            wave_blocks(combine_bwd_kernel<4, true, true>, ntok));
+            gains_smem_ok(combine_bwd_kernel<4, true, false>);
+            gains_smem_ok(combine_bwd_kernel<4, true, true>);
+            return std::max(wave_blocks(combine_bwd_kernel<4, true, false>, ntok, smem),
+                            wave_blocks(combine_bwd_kernel<4, true, true>, ntok, smem));
     }
 }
 
@@ -461,13 +510,15 @@ int combine_bwd_common(const logo_bf16* dO, const logo_bf16* o_l, const logo_bf1
         if (workspace_bytes < logo_combine_bwd_workspace_size(dims)) return LOGO_ERR_WORKSPACE;
     }
     const int64_t ntok = static_cast<int64_t>(dims.B) * dims.T;
+    const size_t smem = gains ? gains_smem(dims) : 0;
     unsigned grid = 0;
     float* part = static_cast<float*>(workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
 #define LOGO_COMBINE_BWD(V, G, U)                                                                                 \
-    grid = static_cast<unsigned>(wave_blocks(combine_bwd_kernel<V, G, U>, ntok));                                  \
-    combine_bwd_kernel<V, G, U><<<grid, kThreads, 0, st>>>(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps, dO_l, \
-                                                           dO_c, dgate_p, part, ntok, dims.Hq, dims.D)
+    if (G && !gains_smem_ok(combine_bwd_kernel<V, G, U>)) return LOGO_ERR_CUDA;                                    \
+    grid = static_cast<unsigned>(wave_blocks(combine_bwd_kernel<V, G, U>, ntok, smem));                            \
+    combine_bwd_kernel<V, G, U><<<grid, kThreads, smem, st>>>(dO, o_l, o_c, gate_p, z, row_of, gain_l, gain_g, eps,    \
+                                                              dO_l, dO_c, dgate_p, part, ntok, dims.Hq, dims.D)
     const bool unit = !gain_l && !gain_g;
     if (gains && unit) {
         switch (vpt) {

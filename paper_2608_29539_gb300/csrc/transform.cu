@@ -61,52 +61,90 @@ __device__ __forceinline__ uint32_t toff(int row, int chunk)
     return static_cast<uint32_t>(row * (D * 2) + ((chunk ^ (row & 7)) << 4));
 }
 
-// Load rows [0, nrows) of a tile (token indices in tok[]) of head h; rows past
-// the end are zero.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wait_group 1;\n" ::: "memory"); }
+
+__device__ __forceinline__ void st_shared_b32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
+}
+
+// Start the copies of rows [0, nrows) of a tile (token indices in tok[]) of
+// head h into shared memory; rows past the end are zeroed with plain stores.
+// The copies complete at the caller's cp.async wait.
 template <int D>
-__device__ __forceinline__ void load_tile(uint32_t dst, const logo_bf16* src, const int64_t* tok, int nrows, int H,
-                                          int h, int nthreads)
+__device__ __forceinline__ void load_tile_async(uint32_t dst, const logo_bf16* src, const int64_t* tok, int nrows,
+                                                int H, int h, int nthreads)
 {
     constexpr int kChunks = D / 8;
     for (int idx = threadIdx.x; idx < kTileRows * kChunks; idx += nthreads) {
         const int r = idx / kChunks, c = idx % kChunks;
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (r < nrows) v = *reinterpret_cast<const uint4*>(src + (tok[r] * H + h) * D + c * 8);
-        st_shared_v4(dst + toff<D>(r, c), v.x, v.y, v.z, v.w);
+        if (r < nrows) cp_async16(dst + toff<D>(r, c), src + (tok[r] * H + h) * D + c * 8);
+        else st_shared_v4(dst + toff<D>(r, c), 0u, 0u, 0u, 0u);
     }
 }
 
 template <int D>
-__device__ __forceinline__ void load_matrix(uint32_t dst, const logo_bf16* a, int nthreads)
+__device__ __forceinline__ void load_matrix_async(uint32_t dst, const logo_bf16* a, int nthreads)
 {
     constexpr int kChunks = D / 8;
     for (int idx = threadIdx.x; idx < D * kChunks; idx += nthreads) {
         const int r = idx / kChunks, c = idx % kChunks;
-        const uint4 v = *reinterpret_cast<const uint4*>(a + r * D + c * 8);
-        st_shared_v4(dst + toff<D>(r, c), v.x, v.y, v.z, v.w);
+        cp_async16(dst + toff<D>(r, c), a + r * D + c * 8);
     }
 }
 
-// LP forward: u_g[row] = u_l[row] A_h.  4 warps, 16 rows of the 64-row tile each.
+// token index of row r of the listed set, 0 past the end
+__device__ __forceinline__ int64_t tile_token(const RowSet& R, int n, int r) { return r < n ? row_token(R, r) : 0; }
+
+// LP forward: u_g[row] = u_l[row] A_h.  4 warps, 16 rows of the 64-row tile
+// each.  A_h and the block's first tile arrive by cp.async together; each later
+// tile is fetched into the second buffer while the current one is multiplied.
+// A warp writes its results back over its own 16 rows of the tile (the only
+// rows its MMAs read), so the stores to global memory leave as whole 2D-byte
+// row pieces, two rows per warp instruction, instead of 16-byte fragments.
 template <int D>
 __global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict__ u_l,
                                                      const logo_bf16* __restrict__ a, RowSet R, int H,
                                                      logo_bf16* __restrict__ u_g)
 {
+    constexpr int kTileBytes = kTileRows * D * 2;
+    constexpr int kChunks = D / 8;
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ int64_t tok[kTileRows];
+    __shared__ int64_t tok[2][kTileRows];
     const uint32_t sA = smem_u32(smem), sU = sA + D * D * 2;
     const int h = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int mi = lane >> 3, rr = lane & 7, gid = lane >> 2, tig = lane & 3;
-    load_matrix<D>(sA, a + static_cast<int64_t>(h) * D * D, 128);
     const int n = row_count(R);
     const int ntiles = (n + kTileRows - 1) / kTileRows;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int r0 = tile * kTileRows, nr = min(kTileRows, n - r0);
-        if (threadIdx.x < kTileRows) tok[threadIdx.x] = threadIdx.x < nr ? row_token(R, r0 + threadIdx.x) : 0;
+    int tile = blockIdx.x;
+    if (tile >= ntiles) return;
+    load_matrix_async<D>(sA, a + static_cast<int64_t>(h) * D * D, 128);
+    if (threadIdx.x < kTileRows) tok[0][threadIdx.x] = tile_token(R, n, tile * kTileRows + threadIdx.x);
+    __syncthreads();
+    load_tile_async<D>(sU, u_l, tok[0], min(kTileRows, n - tile * kTileRows), H, h, 128);
+    cp_async_commit();
+    for (int k = 0; tile < ntiles; tile += gridDim.x, ++k) {
+        const int buf = k & 1;
+        const int nr = min(kTileRows, n - tile * kTileRows);
+        const int next = tile + gridDim.x;
+        if (next < ntiles) {  // the buffer and token list of tile k-1 are free (barrier at the loop's end)
+            if (threadIdx.x < kTileRows) tok[buf ^ 1][threadIdx.x] = tile_token(R, n, next * kTileRows + threadIdx.x);
+            __syncthreads();
+            load_tile_async<D>(sU + (buf ^ 1) * kTileBytes, u_l, tok[buf ^ 1], min(kTileRows, n - next * kTileRows),
+                               H, h, 128);
+            cp_async_commit();
+            cp_async_wait_one();
+        } else {
+            cp_async_wait_all();
+        }
         __syncthreads();
-        load_tile<D>(sU, u_l, tok, nr, H, h, 128);
-        __syncthreads();
+        const uint32_t sT = sU + buf * kTileBytes;
         float acc[D / 8][4];
 #pragma unroll
         for (int nt = 0; nt < D / 8; ++nt)
@@ -115,7 +153,7 @@ __global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict
 #pragma unroll
         for (int ks = 0; ks < D / 16; ++ks) {
             uint32_t fa[4];
-            ldsm_x4(sU + toff<D>(warp * 16 + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), fa[0], fa[1], fa[2], fa[3]);
+            ldsm_x4(sT + toff<D>(warp * 16 + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), fa[0], fa[1], fa[2], fa[3]);
 #pragma unroll
             for (int np = 0; np < D / 16; ++np) {
                 uint32_t b0, b1, b2, b3;  // A_h rows k (input dim), columns n (output dim)
@@ -124,14 +162,21 @@ __global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict
                 mma_bf16_16816(acc[2 * np + 1], fa, b2, b3);
             }
         }
+        __syncwarp();
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
             const int r = warp * 16 + gid + half * 8;
-            if (r < nr) {
-                logo_bf16* dst = u_g + (tok[r] * H + h) * D + 2 * tig;
 #pragma unroll
-                for (int nt = 0; nt < D / 8; ++nt)
-                    *reinterpret_cast<uint32_t*>(dst + nt * 8) = pack_bf16x2(acc[nt][2 * half], acc[nt][2 * half + 1]);
+            for (int nt = 0; nt < D / 8; ++nt)
+                st_shared_b32(sT + toff<D>(r, nt) + 4 * tig, pack_bf16x2(acc[nt][2 * half], acc[nt][2 * half + 1]));
+        }
+        __syncwarp();
+#pragma unroll
+        for (int idx = lane; idx < 16 * kChunks; idx += 32) {
+            const int r = warp * 16 + idx / kChunks, c = idx % kChunks;
+            if (r < nr) {
+                const uint4 v = ld_shared_v4(sT + toff<D>(r, c));
+                *reinterpret_cast<uint4*>(u_g + (tok[buf][r] * H + h) * D + c * 8) = v;
             }
         }
         __syncthreads();
@@ -155,7 +200,7 @@ __global__ void __launch_bounds__(D * 2) lp_bwd_kernel(const logo_bf16* __restri
     const uint32_t sA = smem_u32(smem), sU = sA + D * D * 2, sG = sU + kTileRows * D * 2;
     const int h = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int mi = lane >> 3, rr = lane & 7, gid = lane >> 2, tig = lane & 3;
-    load_matrix<D>(sA, a + static_cast<int64_t>(h) * D * D, kThreads);
+    load_matrix_async<D>(sA, a + static_cast<int64_t>(h) * D * D, kThreads);  // lands with the first tile
     float acc_a[D / 8][4];
 #pragma unroll
     for (int nt = 0; nt < D / 8; ++nt)
@@ -168,8 +213,10 @@ __global__ void __launch_bounds__(D * 2) lp_bwd_kernel(const logo_bf16* __restri
         const int r0 = tile * kTileRows, nr = min(kTileRows, n - r0);
         if (threadIdx.x < kTileRows) tok[threadIdx.x] = threadIdx.x < nr ? row_token(R, r0 + threadIdx.x) : 0;
         __syncthreads();
-        load_tile<D>(sU, u_l, tok, nr, H, h, kThreads);
-        load_tile<D>(sG, du_g, tok, nr, H, h, kThreads);
+        load_tile_async<D>(sU, u_l, tok, nr, H, h, kThreads);
+        load_tile_async<D>(sG, du_g, tok, nr, H, h, kThreads);
+        cp_async_commit();
+        cp_async_wait_all();
         __syncthreads();
         // dU = dG A^T: rows 16 rg.., output columns cb .. cb + 63 (A_h rows i)
         {
@@ -224,6 +271,7 @@ __global__ void __launch_bounds__(D * 2) lp_bwd_kernel(const logo_bf16* __restri
         }
         __syncthreads();
     }
+    cp_async_wait_all();  // a block with no tile still has A_h's copies in flight
     float* pp = part + (static_cast<int64_t>(h) * gridDim.x + blockIdx.x) * D * D;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -765,9 +813,14 @@ template <int D>
 int launch_lp_fwd(const logo_bf16* u_l, const logo_bf16* a, const RowSet& R, int H, logo_bf16* u_g,
                   cudaStream_t st)
 {
-    const int smem = D * D * 2 + kTileRows * D * 2;
+    const int smem = D * D * 2 + 2 * kTileRows * D * 2;  // A_h and two row tiles
     if (set_smem_limit(lp_fwd_kernel<D>, smem) != cudaSuccess) return LOGO_ERR_CUDA;
-    lp_fwd_kernel<D><<<dim3(kChunksPerHead, H), 128, smem, st>>>(u_l, a, R, H, u_g);
+    // one wave: blocks per SM as shared memory allows (3 at d = 128, 64 KB each),
+    // split evenly over the heads; each block walks a strided share of its head's tiles
+    const int per_sm = D == 128 ? 3 : 6;
+    int chunks = per_sm * device_sm_count() / H;
+    chunks = chunks < 1 ? 1 : chunks > 64 ? 64 : chunks;
+    lp_fwd_kernel<D><<<dim3(chunks, H), 128, smem, st>>>(u_l, a, R, H, u_g);
     return cudaGetLastError() == cudaSuccess ? LOGO_OK : LOGO_ERR_CUDA;
 }
 

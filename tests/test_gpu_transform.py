@@ -45,6 +45,11 @@ CASES = [
     (1, 1000, 2, 64, None),
     (3, 257, 3, 64, 0.5),
     (2, 2048, 32, 128, 0.125),   # several tiles per block, the 16K workload's head count
+    # more row tiles per head than blocks per head: the selected-row LP forward
+    # fetches a block's next tile while it multiplies the current one (both
+    # buffers in use), with a ragged last tile
+    (1, 8100, 32, 128, 0.25),
+    (1, 16000, 16, 64, 0.25),
 ]
 
 
