@@ -103,8 +103,10 @@ __device__ __forceinline__ void load_matrix_async(uint32_t dst, const logo_bf16*
 __device__ __forceinline__ int64_t tile_token(const RowSet& R, int n, int r) { return r < n ? row_token(R, r) : 0; }
 
 // LP forward: u_g[row] = u_l[row] A_h.  4 warps, 16 rows of the 64-row tile
-// each.  A_h and the block's first tile arrive by cp.async together; each later
-// tile is fetched into the second buffer while the current one is multiplied.
+// each.  A block walks a strided share of its head's row tiles with two tile
+// buffers: the copies of A_h start before the row count is read, the token
+// lists of the first two tiles are looked up together, and tile k+2 is
+// fetched (cp.async) while tile k+1 is in flight and tile k is multiplied.
 // A warp writes its results back over its own 16 rows of the tile (the only
 // rows its MMAs read), so the stores to global memory leave as whole 2D-byte
 // row pieces, two rows per warp instruction, instead of 16-byte fragments.
@@ -120,29 +122,31 @@ __global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict
     const uint32_t sA = smem_u32(smem), sU = sA + D * D * 2;
     const int h = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int mi = lane >> 3, rr = lane & 7, gid = lane >> 2, tig = lane & 3;
+    load_matrix_async<D>(sA, a + static_cast<int64_t>(h) * D * D, 128);  // joins the first tile's group
     const int n = row_count(R);
     const int ntiles = (n + kTileRows - 1) / kTileRows;
+    const int step = gridDim.x;
     int tile = blockIdx.x;
-    if (tile >= ntiles) return;
-    load_matrix_async<D>(sA, a + static_cast<int64_t>(h) * D * D, 128);
-    if (threadIdx.x < kTileRows) tok[0][threadIdx.x] = tile_token(R, n, tile * kTileRows + threadIdx.x);
+    if (tile >= ntiles) {  // no tile: let A_h's copies land before the block exits
+        cp_async_wait_all();
+        return;
+    }
+    {  // threads 0..63: rows of the first tile, 64..127: rows of the second
+        const int which = threadIdx.x / kTileRows, r = threadIdx.x % kTileRows;
+        tok[which][r] = tile_token(R, n, (tile + which * step) * kTileRows + r);
+    }
     __syncthreads();
     load_tile_async<D>(sU, u_l, tok[0], min(kTileRows, n - tile * kTileRows), H, h, 128);
     cp_async_commit();
-    for (int k = 0; tile < ntiles; tile += gridDim.x, ++k) {
+    if (tile + step < ntiles) {
+        load_tile_async<D>(sU + kTileBytes, u_l, tok[1], min(kTileRows, n - (tile + step) * kTileRows), H, h, 128);
+        cp_async_commit();
+    }
+    for (int k = 0; tile < ntiles; tile += step, ++k) {
         const int buf = k & 1;
         const int nr = min(kTileRows, n - tile * kTileRows);
-        const int next = tile + gridDim.x;
-        if (next < ntiles) {  // the buffer and token list of tile k-1 are free (barrier at the loop's end)
-            if (threadIdx.x < kTileRows) tok[buf ^ 1][threadIdx.x] = tile_token(R, n, next * kTileRows + threadIdx.x);
-            __syncthreads();
-            load_tile_async<D>(sU + (buf ^ 1) * kTileBytes, u_l, tok[buf ^ 1], min(kTileRows, n - next * kTileRows),
-                               H, h, 128);
-            cp_async_commit();
-            cp_async_wait_one();
-        } else {
-            cp_async_wait_all();
-        }
+        if (tile + step < ntiles) cp_async_wait_one();  // tile k+1 may stay in flight
+        else cp_async_wait_all();
         __syncthreads();
         const uint32_t sT = sU + buf * kTileBytes;
         float acc[D / 8][4];
@@ -179,7 +183,14 @@ __global__ void __launch_bounds__(128) lp_fwd_kernel(const logo_bf16* __restrict
                 *reinterpret_cast<uint4*>(u_g + (tok[buf][r] * H + h) * D + c * 8) = v;
             }
         }
-        __syncthreads();
+        __syncthreads();  // buffer buf and tok[buf] are free
+        const int after = tile + 2 * step;  // tile k+2 goes where tile k was
+        if (after < ntiles) {
+            if (threadIdx.x < kTileRows) tok[buf][threadIdx.x] = tile_token(R, n, after * kTileRows + threadIdx.x);
+            __syncthreads();
+            load_tile_async<D>(sT, u_l, tok[buf], min(kTileRows, n - after * kTileRows), H, h, 128);
+            cp_async_commit();
+        }
     }
 }
 
