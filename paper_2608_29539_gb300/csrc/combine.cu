@@ -77,29 +77,6 @@ __device__ __forceinline__ Vec8 load_gain(const float* g, int h, int D, int j)
     return r;
 }
 
-// sum_i x_i^2 and sum_i x_i y_i over a vector of 8, as f32x2 pairs
-__device__ __forceinline__ float sumsq8(const Vec8& x)
-{
-    uint64_t a = f2_mul(f2_pack(x.v[0], x.v[1]), f2_pack(x.v[0], x.v[1]));
-    uint64_t b = f2_mul(f2_pack(x.v[2], x.v[3]), f2_pack(x.v[2], x.v[3]));
-    a = f2_fma(f2_pack(x.v[4], x.v[5]), f2_pack(x.v[4], x.v[5]), a);
-    b = f2_fma(f2_pack(x.v[6], x.v[7]), f2_pack(x.v[6], x.v[7]), b);
-    float lo, hi;
-    f2_unpack(f2_add(a, b), lo, hi);
-    return lo + hi;
-}
-
-__device__ __forceinline__ float dot8(const Vec8& x, const Vec8& y)
-{
-    uint64_t a = f2_mul(f2_pack(x.v[0], x.v[1]), f2_pack(y.v[0], y.v[1]));
-    uint64_t b = f2_mul(f2_pack(x.v[2], x.v[3]), f2_pack(y.v[2], y.v[3]));
-    a = f2_fma(f2_pack(x.v[4], x.v[5]), f2_pack(y.v[4], y.v[5]), a);
-    b = f2_fma(f2_pack(x.v[6], x.v[7]), f2_pack(y.v[6], y.v[7]), b);
-    float lo, hi;
-    f2_unpack(f2_add(a, b), lo, hi);
-    return lo + hi;
-}
-
 // x * a + y * b elementwise (y, b optional), as f32x2 pairs
 __device__ __forceinline__ Vec8 axpby8(const Vec8& x, float a, const Vec8* y, float b)
 {
